@@ -1,0 +1,415 @@
+#!/usr/bin/env python
+"""Decode throughput of the KVpop hot path on GB300.
+
+One "step" = one decode step of the whole batch through the C ABI: ingest the
+new token, delayed scorer on the token leaving the window, keep-or-drop
+eviction, scatter (kvpop_decode_ingest) and GQA decode attention over the
+compressed cache (kvpop_decode_attend).  Prefill is done once, untimed.
+
+Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle instead
+(the reference arm: the paper publishes no code and no decode throughput).
+Under torchrun (N > 1) every rank runs an independent replica of the workload
+(the path has no cross-sequence exchange); value = all ranks' tokens / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/sec at 1 GB300 (batch x steps) and achieved HBM GB/s"
+DEFAULT_CONFIG = "cr8x"
+ATTEND_SRC = os.path.join(ROOT, "paper_2607_05061_gb300", "csrc", "kvpop_attend.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attend_kernel_traffic.txt")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2048)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["kvpop", "reference"], default="kvpop")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--e2e-steps", type=int, default=256)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-steps", type=int, default=96)
+    return ap.parse_args(argv)
+
+
+# ------------------------------------------------------------------ distributed plumbing
+def dist_info():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def dist_init(world, backend):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def reduce_max_sum(local_max: float, local_sum: float, world: int, device=None):
+    """(max over ranks of local_max, sum over ranks of local_sum)."""
+    if world <= 1:
+        return local_max, local_sum
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([local_max], dtype=torch.float64, device=device)
+    s = torch.tensor([local_sum], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(s, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(s.item())
+
+
+# ------------------------------------------------------------------ workload arithmetic
+def kv_stream_bytes(cfg, lengths, step: int) -> int:
+    """Algorithmic K/V bytes one attention launch reads at decode step `step` (0-based).
+
+    Per (sequence, KV head): (used slots + window entries) * 2 (K and V) * d * esz,
+    with len = P + step + 1 after the step's token is ingested.
+    """
+    tot = 0
+    for P in lengths:
+        ln = P + step + 1
+        keys = min(cfg.budget_B, max(0, ln - cfg.delay_D)) + min(ln, cfg.delay_D)
+        tot += keys
+    return tot * cfg.n_kv_heads * 2 * cfg.head_dim * cfg.esz
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def committed_traffic(config_name: str):
+    """DRAM bytes per attention launch from the committed ncu summary, if it matches the source."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    kv = {}
+    with open(TRAFFIC_FILE) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 2 and not line.startswith("#"):
+                kv[parts[0]] = parts[1]
+    sha = hashlib.sha256(open(ATTEND_SRC, "rb").read()).hexdigest()
+    if kv.get("source_sha256") != sha or kv.get("config") != config_name:
+        return None
+    try:
+        return int(float(kv["dram_bytes_per_launch"]))
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples taken while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                cols = [c.strip() for c in line.split(",")]
+                if len(cols) >= 9:
+                    rows.append(cols)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ oracle (CPU) legs
+def _oracle_pair_job(args):
+    """Prefill one (sequence, KV head) in the oracle (untimed), then time n decode steps."""
+    cfg_name, b, h, n_steps = args
+    import torch
+    torch.set_num_threads(1)
+    from oracle.run import prefill_pair
+    from workload import gen, get_config
+    cfg = get_config(cfg_name)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    cache = prefill_pair(cfg, w, b, h, L[b])
+    G = cfg.q_per_kv
+    q, k, v = gen.decode_inputs(cfg, [L[b]], 0, n_steps, b0=b)
+    q = q[:, 0, h * G:(h + 1) * G].double().numpy()
+    k = k[:, 0, h].double().numpy()
+    v = v[:, 0, h].double().numpy()
+    t0 = time.perf_counter()
+    for j in range(n_steps):
+        cache.append(q[j], k[j], v[j])
+        cache.attend(q[j])
+    return time.perf_counter() - t0
+
+
+def sample_pairs(cfg, n):
+    total = cfg.batch * cfg.n_kv_heads
+    idx = sorted({(i * total) // n for i in range(n)})
+    return [(i // cfg.n_kv_heads, i % cfg.n_kv_heads) for i in idx]
+
+
+def cpu_baseline(cfg, n_steps: int):
+    """fp64 oracle decode throughput on this host's cores (spawned pool, one pair per core)."""
+    import multiprocessing as mp
+    cores = max(1, min(os.cpu_count() or 1, 16))
+    pairs = sample_pairs(cfg, cores)
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(len(pairs)) as pool:
+        times = pool.map(_oracle_pair_job, [(cfg.name, b, h, n_steps) for b, h in pairs])
+    per_pair_step = statistics.mean(times) / n_steps            # seconds per (pair, step)
+    step_time = cfg.batch * cfg.n_kv_heads * per_pair_step / len(pairs)
+    return {"value": cfg.batch / step_time, "unit": "tokens/s", "cores": len(pairs), "kind": "oracle",
+            "sample": (f"{len(pairs)} of {cfg.batch * cfg.n_kv_heads} (sequence, KV head) pairs, "
+                       f"{n_steps} decode steps each after an untimed oracle prefill, one pair per "
+                       f"core in parallel; whole-batch step time extrapolated as pairs/cores x "
+                       f"mean pair-step time")}
+
+
+# ------------------------------------------------------------------ GPU arm
+def run_kvpop(args):
+    import torch
+    rank, local_rank, world = dist_info()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = dist_init(world, "nccl")
+
+    from paper_2607_05061_gb300 import build as _build
+    _build.build()
+    from paper_2607_05061_gb300 import kvpop
+    from workload import gen, get_config
+
+    cfg = get_config(args.config)
+    if cfg.n_layers != 1:
+        raise SystemExit("bench.py times single-layer workloads (tiny, q4b, cr8x, ragged)")
+    L = gen.prompt_lengths(cfg)
+    W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
+    cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
+                             cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
+                             n_sink=cfg.n_sink)
+    # prefill (untimed), a few sequences at a time to bound the prompt buffers
+    group = 8
+    for b0 in range(0, cfg.batch, group):
+        nb = min(group, cfg.batch - b0)
+        Lg = L[b0:b0 + nb]
+        Pm = max(Lg)
+        Q = gen.q_tokens(cfg, b0, nb, 0, Pm, device=dev)
+        K = gen.kv_tokens(cfg, "k", b0, nb, 0, Pm, device=dev)
+        V = gen.kv_tokens(cfg, "v", b0, nb, 0, Pm, device=dev)
+        cache.prefill(Q, K, V, Lg, first_seq=b0)
+        del Q, K, V
+    torch.cuda.synchronize()
+
+    W, K = args.warmup, args.steps
+    q, k, v = gen.decode_inputs(cfg, L, 0, W + K, device=dev)
+    out = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    for j in range(W):
+        cache.ingest(q[j], k[j], v[j])
+        cache.attend(q[j], out)
+    torch.cuda.synchronize()
+
+    ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(K):
+        j = W + i
+        cache.ingest(q[j], k[j], v[j])
+        ev_s[i].record(stream)
+        cache.attend(q[j], out)
+        ev_e[i].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    cache.check()
+    step_ms_local = t_start.elapsed_time(t_end) / K
+    attn_ms = statistics.mean(ev_s[i].elapsed_time(ev_e[i]) for i in range(K))
+
+    # end to end through the C ABI on host buffers (pinned), copies inside the timed region
+    E = max(1, args.e2e_steps)
+    qh, kh, vh = gen.decode_inputs(cfg, L, W + K, E, device="cpu")
+    qh, kh, vh = qh.pin_memory(), kh.pin_memory(), vh.pin_memory()
+    outh = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32).pin_memory()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(E):
+        cache.step_host(qh[i], kh[i], vh[i], outh)
+        stream.synchronize()          # the host reads each step's output
+    e2e_s = time.perf_counter() - t0
+    cache.check()
+    h2d = (qh[0].numel() + kh[0].numel() + vh[0].numel()) * qh.element_size()
+    d2h = outh.numel() * 4
+
+    step_ms, _ = reduce_max_sum(step_ms_local, 0.0, world, dev)
+    e2e_max, _ = reduce_max_sum(e2e_s / E * 1e3, 0.0, world, dev)
+    tokens_per_step = cfg.batch * world
+    value = tokens_per_step / (step_ms / 1e3)
+    bytes_per_launch = statistics.mean(kv_stream_bytes(cfg, L, W + i) for i in range(K))
+    achieved = bytes_per_launch / (attn_ms / 1e3) / 1e9
+    peak, peak_src = measured_peaks()
+    rec = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded counter-based generator)",
+        "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
+                   "kv_heads": cfg.n_kv_heads, "q_per_kv": cfg.q_per_kv, "head_dim": cfg.head_dim,
+                   "prompt_len": "ragged U[%d,%d]" % cfg.ragged if cfg.ragged else cfg.prompt_len,
+                   "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype,
+                   "scorer": f"MLP {cfg.scorer_in}->{cfg.scorer_hidden} GELU->1 fp32",
+                   "l2": f"inputs larger than L2: {bytes_per_launch / 1e9:.3f} GB K/V read per step",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "steps_per_s": 1e3 / step_ms,
+        "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "attend_kernel", "achieved": achieved, "peak": peak,
+                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                     else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
+                     "frac_of_8tbs_nominal": achieved / 8000.0, "traffic": committed_traffic(cfg.name),
+                     "algorithmic_bytes_per_launch": bytes_per_launch, "ms_per_launch": attn_ms},
+        "e2e": {"value": tokens_per_step / (e2e_max / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": E,
+                "how": "kvpop_decode_step_host on pinned host buffers, stream sync every step"},
+        "gpu_launches": 2 * K,
+        "clocks": clk,
+    }
+    cache.free()
+    del q, k, v
+    if rank == 0 and not args.no_cpu_baseline:
+        rec["cpu_baseline"] = cpu_baseline(cfg, args.cpu_steps)
+    if rank == 0:
+        print(json.dumps(rec), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------ reference arm (oracle)
+def run_reference(args):
+    rank, _, world = dist_info()
+    if rank != 0:
+        return
+    from oracle.run import prefill_pair
+    from workload import gen, get_config
+    cfg = get_config(args.config)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    W, K = args.warmup, args.steps
+    budget_s = 120.0
+    pairs = sample_pairs(cfg, 64)
+    caches, inputs = [], []
+    G = cfg.q_per_kv
+    t_setup = time.perf_counter()
+    for b, h in pairs:
+        caches.append(prefill_pair(cfg, w, b, h, L[b]))
+        q, k, v = gen.decode_inputs(cfg, [L[b]], 0, W + K, b0=b)
+        inputs.append((q[:, 0, h * G:(h + 1) * G].double().numpy(), k[:, 0, h].double().numpy(),
+                       v[:, 0, h].double().numpy()))
+        # bound the sample so the whole run stays within the budget
+        if len(caches) >= 1 and time.perf_counter() - t_setup > 60:
+            break
+    # calibrate: pairs per step so that (W + K) steps take about budget_s
+    c0 = caches[0]
+    t0 = time.perf_counter()
+    qa, ka, va = inputs[0]
+    c0.append(qa[0], ka[0], va[0])
+    c0.attend(qa[0])
+    t_pair = max(time.perf_counter() - t0, 1e-5)
+    n_use = max(1, min(len(caches), int(budget_s / ((W + K) * t_pair))))
+    ptr = [1 if i == 0 else 0 for i in range(len(caches))]
+    times = []
+    for s in range(W + K):
+        t0 = time.perf_counter()
+        for i in range(n_use):
+            qa, ka, va = inputs[i]
+            j = ptr[i]
+            if j >= qa.shape[0]:
+                continue
+            caches[i].append(qa[j], ka[j], va[j])
+            caches[i].attend(qa[j])
+            ptr[i] += 1
+        if s >= W:
+            times.append(time.perf_counter() - t0)
+    step_sample_s = sum(times) / len(times)
+    step_s = step_sample_s * (cfg.batch * cfg.n_kv_heads) / n_use
+    value = cfg.batch / step_s
+    rec = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded counter-based generator)",
+        "impl": "reference",
+        "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
+                   "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": (f"each step = one decode step of {n_use} of "
+                                    f"{cfg.batch * cfg.n_kv_heads} (sequence, KV head) pairs on one "
+                                    f"core after an untimed oracle prefill; whole-batch step time "
+                                    f"extrapolated by pairs")},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(rec), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_kvpop(args)
+
+
+if __name__ == "__main__":
+    main()

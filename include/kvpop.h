@@ -1,0 +1,176 @@
+/*
+ * kvpop.h -- C ABI of the KVpop decode hot path on one GB300 (sm_103a).
+ *
+ * KVpop ("KV cache compression with predictive online pruning") keeps, per KV
+ * head, s sink tokens, a protected window of the w most recent tokens and a
+ * long-range top-k set chosen by a learned scorer (Sec. 3, Eq. 1).  Per decode
+ * step this library
+ *   1. ingests the new token's q/k/v into the window,
+ *   2. scores the token u = p - w that has just left the window with the
+ *      delayed scorer (Sec. 3.3, App. E.4): a two-layer MLP on
+ *      [k_u; v_u; mean of the next w queries of the KV head's query group],
+ *   3. keeps or drops u under the fixed budget (Sec. 3.2 running top-k,
+ *      App. C.1): a free slot while one exists, else it replaces the slot of
+ *      lowest static priority (App. B.3; ties -> lowest slot index) iff its
+ *      priority is strictly larger,
+ *   4. scatters u's K/V into that slot, and
+ *   5. runs GQA decode attention over the compact cache only -- the kept slots
+ *      plus the window (App. C, first paragraph).
+ *
+ * Notation: b = batch, H = KV heads, G = query heads per KV head, d = head
+ * dim, D = window (the paper's w), B = slots (sinks + long-range top-k; the
+ * paper's s + k), F = scorer hidden width.  Query head index = h * G + g.
+ *
+ * Conventions for every call:
+ *  - Pointers named *_dev are device pointers; *_host are host pointers.
+ *    Device pointers must be 16-byte aligned, else KVPOP_ERR_ALIGN.
+ *  - Calls are asynchronous on `stream` unless stated; the caller owns every
+ *    input/output buffer, the library owns the cache.
+ *  - No call aborts or throws; each returns a status.  After a CUDA error the
+ *    cache is poisoned and later calls return KVPOP_ERR_STATE.
+ *  - One cache per attention layer.  Calls on one cache must be serialised
+ *    (one stream, or stream-ordered) -- they share its workspace.
+ */
+#ifndef KVPOP_H
+#define KVPOP_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  KVPOP_OK = 0,
+  KVPOP_ERR_INVALID_ARG = 1,   /* a size or pointer argument is out of range  */
+  KVPOP_ERR_ALIGN = 2,         /* a device pointer is not 16-byte aligned     */
+  KVPOP_ERR_OOM = 3,           /* device allocation failed                    */
+  KVPOP_ERR_CUDA = 4,          /* a CUDA runtime call failed                  */
+  KVPOP_ERR_STATE = 5,         /* cache poisoned by an earlier error, or freed */
+  KVPOP_ERR_DEVICE_CHECK = 6   /* a kernel reported a failed check / timeout  */
+} kvpop_status;
+
+typedef enum { KVPOP_F32 = 0, KVPOP_BF16 = 1 } kvpop_dtype;
+
+typedef struct {
+  int32_t batch;          /* b >= 1                                            */
+  int32_t n_kv_heads;     /* H >= 1                                            */
+  int32_t q_per_kv;       /* G in {1, 2, 4}                                    */
+  int32_t head_dim;       /* d in {64, 128}                                    */
+  int32_t budget_B;       /* B >= 1: sink + long-range slots (Eq. 1: s + k)    */
+  int32_t delay_D;        /* D >= 1: protected window w (Eq. 4); scoring delay */
+  int32_t n_sink;         /* s, 0 <= s < B: first s tokens are never evicted   */
+  int32_t scorer_hidden;  /* F in [1, 1024]; scorer input width is 3 * d       */
+  kvpop_dtype kv_dtype;   /* element type of q, k, v and the K/V store         */
+} kvpop_config;
+
+/* Scorer parameters (Sec. 3.3 / App. E.2 two-layer MLP, GELU(erf) hidden layer).
+ * Host or device fp32 arrays; copied into the cache at init (caller keeps
+ * ownership).  Input order of W1's rows: [k (d); v (d); qbar (d)]. */
+typedef struct {
+  const float* W1;         /* [H][3d][F]                                      */
+  const float* b1;         /* [H][F]                                          */
+  const float* w2;         /* [H][F]                                          */
+  const float* b2;         /* [H]                                             */
+  const float* log_gamma;  /* [H] per-head log decay (App. B.3, n = 1) or NULL
+                              for none; stored priority = r - u * log_gamma   */
+} kvpop_scorer;
+
+typedef struct kvpop_cache kvpop_cache;   /* opaque, library-owned device state */
+
+/* Human-readable name of a status (static string, never NULL). */
+const char* kvpop_status_string(kvpop_status s);
+
+/* Create an empty cache (length 0 for every sequence) on the current device.
+ * Allocates the slot store [b][H][B][d] for K and V, the window rings
+ * [b][H][D][d], per-slot score/position arrays and the attention workspace.
+ * Synchronises `stream` before returning.  *out is NULL on failure. */
+kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* scorer,
+                              cudaStream_t stream, kvpop_cache** out);
+
+/* Release the cache and all its device memory.  kvpop_free(NULL) is KVPOP_OK.
+ * Synchronises the device work of the cache first. */
+kvpop_status kvpop_free(kvpop_cache* cache);
+
+/* Prompt compression (the prefill of the running top-k, Sec. 3.2 / App. C.1).
+ * For sequences first_seq .. first_seq + n_seq - 1, whose prompt lengths are
+ * prompt_len_host[0 .. n_seq-1] (0 <= P <= Pmax), score every token
+ * u <= P - 1 - D with the delayed scorer, keep the s sinks plus the top (B - s)
+ * of the rest by (priority desc, position asc), store them in ascending
+ * position order, and fill the window with the last min(P, D) tokens.
+ * Replaces any state those sequences had.
+ *   Q_dev  [n_seq][H*G][Pmax][d]    K_dev, V_dev [n_seq][H][Pmax][d]
+ *   score_override_dev  [n_seq][H][Pmax] fp32 raw scores used instead of the
+ *                        scorer (entry u), or NULL
+ * Uses a stream-ordered temporary of n_seq*H*Pmax*4 bytes and synchronises
+ * `stream` before returning (the host length array may be reused at once). */
+kvpop_status kvpop_prefill_compress(kvpop_cache* cache, const void* Q_dev, const void* K_dev,
+                                    const void* V_dev, const int32_t* prompt_len_host,
+                                    int32_t first_seq, int32_t n_seq, int32_t Pmax,
+                                    const float* score_override_dev, cudaStream_t stream);
+
+/* Decode steps 1-4 for every sequence: ingest the token at position p = len,
+ * score u = p - D (if p >= D), keep or drop it, scatter it, push p.
+ *   q_dev [b][H*G][d], k_dev / v_dev [b][H][d]
+ *   score_override_dev [b][H] fp32 raw scores used instead of the scorer, or NULL
+ *   evict_info_dev [b][H][2] int32 out: (slot u went to or -1, evicted position
+ *                  or -1), or NULL
+ *   score_out_dev  [b][H] fp32 out: raw score of u (NaN when no token left the
+ *                  window), or NULL */
+kvpop_status kvpop_decode_ingest(kvpop_cache* cache, const void* q_dev, const void* k_dev,
+                                 const void* v_dev, const float* score_override_dev,
+                                 int32_t* evict_info_dev, float* score_out_dev,
+                                 cudaStream_t stream);
+
+/* Decode step 5: out_g = softmax(q_g K_S^T / sqrt(d)) V_S for every query head,
+ * where S = kept slots plus window entries of its KV head.  Split-K over a
+ * persistent grid with token-balanced ranges.
+ *   q_dev [b][H*G][d] (same as ingest)   out_dev [b][H*G][d] fp32 */
+kvpop_status kvpop_decode_attend(kvpop_cache* cache, const void* q_dev, float* out_dev,
+                                 cudaStream_t stream);
+
+/* kvpop_decode_ingest followed by kvpop_decode_attend. */
+kvpop_status kvpop_decode_step(kvpop_cache* cache, const void* q_dev, const void* k_dev,
+                               const void* v_dev, float* out_dev,
+                               const float* score_override_dev, int32_t* evict_info_dev,
+                               float* score_out_dev, cudaStream_t stream);
+
+/* kvpop_decode_step on host buffers (pinned memory recommended): copies q/k/v
+ * into library-owned device staging, runs the step and copies out back, all
+ * on `stream` (the caller synchronises before reading out_host). */
+kvpop_status kvpop_decode_step_host(kvpop_cache* cache, const void* q_host, const void* k_host,
+                                    const void* v_host, float* out_host, cudaStream_t stream);
+
+/* Synchronise `stream` and report any device-side check failure
+ * (KVPOP_ERR_DEVICE_CHECK) or CUDA error recorded since the last call. */
+kvpop_status kvpop_check(kvpop_cache* cache, cudaStream_t stream);
+
+/* Checkpoint / resume.  kvpop_export_state with host_buf == NULL sets *bytes to
+ * the size needed; otherwise it copies the full cache state (including lengths)
+ * into host_buf (*bytes >= size) and synchronises.  kvpop_import_state restores
+ * a blob exported from a cache with an identical config. */
+kvpop_status kvpop_export_state(kvpop_cache* cache, void* host_buf, size_t* bytes,
+                                cudaStream_t stream);
+kvpop_status kvpop_import_state(kvpop_cache* cache, const void* host_buf, size_t bytes,
+                                cudaStream_t stream);
+
+/* Per-sequence lengths (tokens seen so far) copied to host; synchronises. */
+kvpop_status kvpop_get_lengths(kvpop_cache* cache, int32_t* len_host, cudaStream_t stream);
+
+/* Diagnostic read of one (sequence, KV head): the positions held by its B
+ * slots (pos_host[B], -1 = free) and their stored priorities (score_host[B];
+ * either may be NULL), and its number of used slots.  Synchronises. */
+kvpop_status kvpop_get_pair_state(kvpop_cache* cache, int32_t seq, int32_t head,
+                                  int32_t* pos_host, float* score_host, int32_t* nvalid_host,
+                                  cudaStream_t stream);
+
+/* Testing hook: make the n-th device allocation from now fail (n >= 1), or
+ * disable with n <= 0.  Affects only this library's allocations. */
+void kvpop_debug_fail_alloc_after(int32_t n);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVPOP_H */

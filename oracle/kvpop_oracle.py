@@ -114,6 +114,7 @@ class HeadCache:
         self.n_valid = 0
         self.pending = deque()      # (pos, k[d], v[d], qmean[d]) oldest first
         self.length = 0
+        self.prefill_raw = np.zeros(0, dtype=np.float32)
 
     # ---- Sec. 3.3 delayed scorer input -------------------------------------------------
     def scorer_input(self, qmean_p: np.ndarray):
@@ -237,6 +238,7 @@ def prefill_head(p: OracleParams, Q: np.ndarray, K: np.ndarray, V: np.ndarray,
         c.slot_raw[slot] = raw[u]
         c.slot_pos[slot] = u
     c.n_valid = len(kept)
+    c.prefill_raw = raw            # fp32 raw score of every eligible prompt token
     for t in range(max(0, P - D), P):
         c.pending.append((t, K[t].copy(), V[t].copy(), qmean[t].copy()))
     c.length = P

@@ -1,0 +1,426 @@
+// Host side of the C ABI declared in include/kvpop.h: argument checks, device
+// memory, kernel launches.  No call throws or aborts; every failure is a status.
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "kvpop_internal.cuh"
+
+using namespace kvpop;
+
+namespace kvpop {
+cudaError_t prepare_ingest(const Dims& dm);
+cudaError_t prepare_prefill(const Dims& dm);
+}
+
+struct kvpop_cache {
+  kvpop_config cfg;
+  Dims dm;
+  State st;
+  int device = 0;
+  int attend_grid = 0;
+  size_t esz = 0;
+  bool poisoned = false;
+  bool has_decay = false;
+  std::vector<void*> allocs;
+  // staging for kvpop_decode_step_host
+  void* stage_q = nullptr;
+  void* stage_k = nullptr;
+  void* stage_v = nullptr;
+  float* stage_out = nullptr;
+  uint64_t magic = 0;
+};
+
+namespace {
+
+constexpr uint64_t kMagic = 0x6b7670'6f70'6361ull;   // "kvpopca"
+constexpr uint64_t kStateVersion = 1;
+int g_fail_after = 0;
+
+kvpop_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return KVPOP_OK;
+  if (e == cudaErrorMemoryAllocation) return KVPOP_ERR_OOM;
+  return KVPOP_ERR_CUDA;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+kvpop_status dev_alloc(kvpop_cache* c, void** p, size_t bytes) {
+  *p = nullptr;
+  if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();   // clear the sticky-free allocation error
+    *p = nullptr;
+    return from_cuda(e);
+  }
+  c->allocs.push_back(*p);
+  return KVPOP_OK;
+}
+
+void release(kvpop_cache* c) {
+  for (void* p : c->allocs) cudaFree(p);
+  c->allocs.clear();
+}
+
+kvpop_status validate(const kvpop_config* cfg) {
+  if (!cfg) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->batch < 1 || cfg->n_kv_heads < 1) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->q_per_kv != 1 && cfg->q_per_kv != 2 && cfg->q_per_kv != 4) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->head_dim != 64 && cfg->head_dim != 128) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->budget_B < 1 || cfg->delay_D < 1) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->n_sink < 0 || cfg->n_sink >= cfg->budget_B) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->scorer_hidden < 1 || cfg->scorer_hidden > 1024) return KVPOP_ERR_INVALID_ARG;
+  if (cfg->kv_dtype != KVPOP_F32 && cfg->kv_dtype != KVPOP_BF16) return KVPOP_ERR_INVALID_ARG;
+  const long long pairs = (long long)cfg->batch * cfg->n_kv_heads;
+  if (pairs > 12288) return KVPOP_ERR_INVALID_ARG;             // attention schedule in smem
+  if ((long long)cfg->budget_B * pairs > (1ll << 40)) return KVPOP_ERR_INVALID_ARG;
+  return KVPOP_OK;
+}
+
+kvpop_status usable(kvpop_cache* c) {
+  if (!c || c->magic != kMagic) return KVPOP_ERR_INVALID_ARG;
+  if (c->poisoned) return KVPOP_ERR_STATE;
+  return KVPOP_OK;
+}
+
+kvpop_status poison_on(kvpop_cache* c, cudaError_t e) {
+  if (e == cudaSuccess) return KVPOP_OK;
+  c->poisoned = true;
+  return from_cuda(e);
+}
+
+struct StateBuf {
+  void* ptr;
+  size_t bytes;
+};
+
+std::vector<StateBuf> state_buffers(kvpop_cache* c) {
+  const Dims& dm = c->dm;
+  const size_t pairs = dm.pairs;
+  return {
+      {c->st.slotK, pairs * dm.B * dm.d * c->esz},
+      {c->st.slotV, pairs * dm.B * dm.d * c->esz},
+      {c->st.ringK, pairs * dm.D * dm.d * c->esz},
+      {c->st.ringV, pairs * dm.D * dm.d * c->esz},
+      {c->st.ringQm, pairs * dm.D * dm.d * 4},
+      {c->st.score, pairs * dm.B * 4},
+      {c->st.pos, pairs * dm.B * 4},
+      {c->st.nvalid, pairs * 4},
+      {c->st.len, pairs * 4},
+      {c->st.min_score, pairs * 4},
+      {c->st.min_slot, pairs * 4},
+  };
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* kvpop_status_string(kvpop_status s) {
+  switch (s) {
+    case KVPOP_OK: return "ok";
+    case KVPOP_ERR_INVALID_ARG: return "invalid argument";
+    case KVPOP_ERR_ALIGN: return "device pointer not 16-byte aligned";
+    case KVPOP_ERR_OOM: return "device allocation failed";
+    case KVPOP_ERR_CUDA: return "CUDA runtime error";
+    case KVPOP_ERR_STATE: return "cache unusable after an earlier error";
+    case KVPOP_ERR_DEVICE_CHECK: return "device-side check failed";
+  }
+  return "unknown status";
+}
+
+void kvpop_debug_fail_alloc_after(int32_t n) { g_fail_after = n > 0 ? n : 0; }
+
+kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
+                              cudaStream_t stream, kvpop_cache** out) {
+  if (!out) return KVPOP_ERR_INVALID_ARG;
+  *out = nullptr;
+  kvpop_status vs = validate(cfg);
+  if (vs != KVPOP_OK) return vs;
+  if (!sc || !sc->W1 || !sc->b1 || !sc->w2 || !sc->b2) return KVPOP_ERR_INVALID_ARG;
+
+  kvpop_cache* c = new (std::nothrow) kvpop_cache();
+  if (!c) return KVPOP_ERR_OOM;
+  c->cfg = *cfg;
+  Dims& dm = c->dm;
+  dm.batch = cfg->batch; dm.H = cfg->n_kv_heads; dm.G = cfg->q_per_kv; dm.d = cfg->head_dim;
+  dm.B = cfg->budget_B; dm.D = cfg->delay_D; dm.s = cfg->n_sink; dm.F = cfg->scorer_hidden;
+  dm.dtype = cfg->kv_dtype;
+  dm.pairs = dm.batch * dm.H;
+  c->esz = cfg->kv_dtype == KVPOP_F32 ? 4 : 2;
+  c->magic = kMagic;
+  cudaGetDevice(&c->device);
+
+  const size_t pairs = dm.pairs, B = dm.B, D = dm.D, d = dm.d, H = dm.H, F = dm.F;
+  const size_t I = 3 * d;
+  AttendConfig ac;
+  kvpop_status s = from_cuda(attend_config(dm, &ac));
+  void* p = nullptr;
+#define ALLOC(field, type, bytes)                        \
+  if (s == KVPOP_OK) {                                   \
+    s = dev_alloc(c, &p, (bytes));                       \
+    c->st.field = static_cast<type>(p);                  \
+  }
+  ALLOC(slotK, void*, pairs * B * d * c->esz)
+  ALLOC(slotV, void*, pairs * B * d * c->esz)
+  ALLOC(ringK, void*, pairs * D * d * c->esz)
+  ALLOC(ringV, void*, pairs * D * d * c->esz)
+  ALLOC(ringQm, float*, pairs * D * d * 4)
+  ALLOC(score, float*, pairs * B * 4)
+  ALLOC(pos, int32_t*, pairs * B * 4)
+  ALLOC(nvalid, int32_t*, pairs * 4)
+  ALLOC(len, int32_t*, pairs * 4)
+  ALLOC(min_score, float*, pairs * 4)
+  ALLOC(min_slot, int32_t*, pairs * 4)
+  float* w = nullptr;
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, (H * I * F + 2 * H * F + 2 * H) * 4); w = (float*)p; }
+  ALLOC(part_count, int32_t*, pairs * 4)
+  ALLOC(err, int32_t*, 16)
+  int sms = 0, occ = 0;
+  if (s == KVPOP_OK) {
+    s = from_cuda(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
+    const size_t smem = ac.smem_fixed + (pairs + 1) * 4;
+    if (s == KVPOP_OK)
+      s = from_cuda(cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    if (s == KVPOP_OK)
+      s = from_cuda(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ac.func, ac.threads, smem));
+    if (s == KVPOP_OK && occ < 1) s = KVPOP_ERR_INVALID_ARG;
+    c->attend_grid = sms * (occ > 0 ? occ : 1);
+  }
+  ALLOC(part, float*, (size_t)2 * c->attend_grid * (dm.G * d + 2 * dm.G) * 4)
+#undef ALLOC
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * c->esz); c->stage_q = p; }
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_k = p; }
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_v = p; }
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * 4); c->stage_out = (float*)p; }
+  if (s == KVPOP_OK) s = from_cuda(prepare_ingest(dm));
+  if (s == KVPOP_OK) s = from_cuda(prepare_prefill(dm));
+  if (s == KVPOP_OK) {
+    float* W1 = w;
+    float* b1 = W1 + H * I * F;
+    float* w2 = b1 + H * F;
+    float* b2 = w2 + H * F;
+    float* lg = b2 + H;
+    c->st.W1 = W1; c->st.b1 = b1; c->st.w2 = w2; c->st.b2 = b2;
+    cudaError_t e = cudaMemcpyAsync(W1, sc->W1, H * I * F * 4, cudaMemcpyDefault, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(b1, sc->b1, H * F * 4, cudaMemcpyDefault, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(w2, sc->w2, H * F * 4, cudaMemcpyDefault, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream);
+    if (e == cudaSuccess && sc->log_gamma) {
+      e = cudaMemcpyAsync(lg, sc->log_gamma, H * 4, cudaMemcpyDefault, stream);
+      c->st.log_gamma = lg;
+      c->has_decay = true;
+    } else {
+      c->st.log_gamma = nullptr;
+    }
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.nvalid, 0, pairs * 4, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.len, 0, pairs * 4, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.part_count, 0, pairs * 4, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.err, 0, 16 * 4, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.pos, 0xff, pairs * B * 4, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    s = from_cuda(e);
+  }
+  if (s != KVPOP_OK) {
+    release(c);
+    c->magic = 0;
+    delete c;
+    return s;
+  }
+  *out = c;
+  return KVPOP_OK;
+}
+
+kvpop_status kvpop_free(kvpop_cache* c) {
+  if (!c) return KVPOP_OK;
+  if (c->magic != kMagic) return KVPOP_ERR_INVALID_ARG;
+  cudaDeviceSynchronize();
+  cudaGetLastError();
+  release(c);
+  c->magic = 0;
+  delete c;
+  return KVPOP_OK;
+}
+
+kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K, const void* V,
+                                    const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
+                                    int32_t Pmax, const float* override_, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!plen_host || n_seq < 0 || first_seq < 0 || first_seq + (long long)n_seq > c->dm.batch ||
+      Pmax < 0 || Pmax > (1 << 24))
+    return KVPOP_ERR_INVALID_ARG;
+  if (n_seq == 0) return KVPOP_OK;
+  for (int i = 0; i < n_seq; ++i)
+    if (plen_host[i] < 0 || plen_host[i] > Pmax) return KVPOP_ERR_INVALID_ARG;
+  if (Pmax > 0 && (!Q || !K || !V)) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(override_))
+    return KVPOP_ERR_ALIGN;
+  const size_t pairs = (size_t)n_seq * c->dm.H;
+  const size_t prio_bytes = pairs * (size_t)Pmax * 4;
+  void* tmp = nullptr;
+  if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
+  cudaError_t e = cudaMallocAsync(&tmp, prio_bytes + 256 + (size_t)n_seq * 4, stream);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return from_cuda(e);
+  }
+  float* prio = static_cast<float*>(tmp);
+  int32_t* plen_dev = reinterpret_cast<int32_t*>(static_cast<char*>(tmp) + ((prio_bytes + 255) & ~size_t(255)));
+  e = cudaMemcpyAsync(plen_dev, plen_host, (size_t)n_seq * 4, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess)
+    e = launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream);
+  // the host copy of the lengths must outlive the async copy
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  cudaError_t e2 = cudaFreeAsync(tmp, stream);
+  if (e == cudaSuccess) e = e2;
+  return poison_on(c, e);
+}
+
+kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, const void* v,
+                                 const float* override_, int32_t* evict_info, float* score_out,
+                                 cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!q || !k || !v) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(override_) ||
+      !aligned16(evict_info) || !aligned16(score_out))
+    return KVPOP_ERR_ALIGN;
+  return poison_on(c, launch_ingest(c->st, c->dm, q, k, v, override_, evict_info, score_out, stream));
+}
+
+kvpop_status kvpop_decode_attend(kvpop_cache* c, const void* q, float* out, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!q || !out) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out)) return KVPOP_ERR_ALIGN;
+  return poison_on(c, launch_attend(c->st, c->dm, q, out, c->attend_grid, stream));
+}
+
+kvpop_status kvpop_decode_step(kvpop_cache* c, const void* q, const void* k, const void* v,
+                               float* out, const float* override_, int32_t* evict_info,
+                               float* score_out, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!out) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(out)) return KVPOP_ERR_ALIGN;
+  s = kvpop_decode_ingest(c, q, k, v, override_, evict_info, score_out, stream);
+  if (s != KVPOP_OK) return s;
+  return kvpop_decode_attend(c, q, out, stream);
+}
+
+kvpop_status kvpop_decode_step_host(kvpop_cache* c, const void* q, const void* k, const void* v,
+                                    float* out, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!q || !k || !v || !out) return KVPOP_ERR_INVALID_ARG;
+  const size_t pairs = c->dm.pairs, d = c->dm.d, G = c->dm.G;
+  cudaError_t e = cudaMemcpyAsync(c->stage_q, q, pairs * G * d * c->esz, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(c->stage_k, k, pairs * d * c->esz, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(c->stage_v, v, pairs * d * c->esz, cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return poison_on(c, e);
+  s = kvpop_decode_step(c, c->stage_q, c->stage_k, c->stage_v, c->stage_out, nullptr, nullptr,
+                        nullptr, stream);
+  if (s != KVPOP_OK) return s;
+  e = cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream);
+  return poison_on(c, e);
+}
+
+kvpop_status kvpop_check(kvpop_cache* c, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return poison_on(c, e);
+  int32_t err[16];
+  e = cudaMemcpy(err, c->st.err, sizeof(err), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return poison_on(c, e);
+  if (err[0] != 0) {
+    cudaMemset(c->st.err, 0, sizeof(err));
+    return KVPOP_ERR_DEVICE_CHECK;
+  }
+  return KVPOP_OK;
+}
+
+kvpop_status kvpop_export_state(kvpop_cache* c, void* host_buf, size_t* bytes, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!bytes) return KVPOP_ERR_INVALID_ARG;
+  auto bufs = state_buffers(c);
+  size_t need = 4 * sizeof(uint64_t) + sizeof(kvpop_config);
+  for (auto& b : bufs) need += b.bytes;
+  if (!host_buf) { *bytes = need; return KVPOP_OK; }
+  if (*bytes < need) { *bytes = need; return KVPOP_ERR_INVALID_ARG; }
+  unsigned char* out = static_cast<unsigned char*>(host_buf);
+  uint64_t hdr[4] = {kMagic, kStateVersion, (uint64_t)need, 0};
+  std::memcpy(out, hdr, sizeof(hdr));
+  std::memcpy(out + sizeof(hdr), &c->cfg, sizeof(kvpop_config));
+  size_t off = sizeof(hdr) + sizeof(kvpop_config);
+  cudaError_t e = cudaSuccess;
+  for (auto& b : bufs) {
+    if (e == cudaSuccess) e = cudaMemcpyAsync(out + off, b.ptr, b.bytes, cudaMemcpyDeviceToHost, stream);
+    off += b.bytes;
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  *bytes = need;
+  return poison_on(c, e);
+}
+
+kvpop_status kvpop_import_state(kvpop_cache* c, const void* host_buf, size_t bytes, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!host_buf) return KVPOP_ERR_INVALID_ARG;
+  const unsigned char* in = static_cast<const unsigned char*>(host_buf);
+  uint64_t hdr[4];
+  if (bytes < sizeof(hdr) + sizeof(kvpop_config)) return KVPOP_ERR_INVALID_ARG;
+  std::memcpy(hdr, in, sizeof(hdr));
+  kvpop_config cfg;
+  std::memcpy(&cfg, in + sizeof(hdr), sizeof(cfg));
+  auto bufs = state_buffers(c);
+  size_t need = sizeof(hdr) + sizeof(kvpop_config);
+  for (auto& b : bufs) need += b.bytes;
+  if (hdr[0] != kMagic || hdr[1] != kStateVersion || hdr[2] != need || bytes < need ||
+      std::memcmp(&cfg, &c->cfg, sizeof(cfg)) != 0)
+    return KVPOP_ERR_INVALID_ARG;
+  size_t off = sizeof(hdr) + sizeof(kvpop_config);
+  cudaError_t e = cudaSuccess;
+  for (auto& b : bufs) {
+    if (e == cudaSuccess) e = cudaMemcpyAsync(b.ptr, in + off, b.bytes, cudaMemcpyHostToDevice, stream);
+    off += b.bytes;
+  }
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->st.part_count, 0, (size_t)c->dm.pairs * 4, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  return poison_on(c, e);
+}
+
+kvpop_status kvpop_get_lengths(kvpop_cache* c, int32_t* len_host, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (!len_host) return KVPOP_ERR_INVALID_ARG;
+  std::vector<int32_t> all((size_t)c->dm.pairs);
+  cudaError_t e = cudaMemcpyAsync(all.data(), c->st.len, all.size() * 4, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return poison_on(c, e);
+  for (int b = 0; b < c->dm.batch; ++b) len_host[b] = all[(size_t)b * c->dm.H];
+  return KVPOP_OK;
+}
+
+kvpop_status kvpop_get_pair_state(kvpop_cache* c, int32_t seq, int32_t head, int32_t* pos_host,
+                                  float* score_host, int32_t* nvalid_host, cudaStream_t stream) {
+  kvpop_status s = usable(c);
+  if (s != KVPOP_OK) return s;
+  if (seq < 0 || seq >= c->dm.batch || head < 0 || head >= c->dm.H) return KVPOP_ERR_INVALID_ARG;
+  const size_t pair = (size_t)seq * c->dm.H + head, B = c->dm.B;
+  cudaError_t e = cudaSuccess;
+  if (pos_host) e = cudaMemcpyAsync(pos_host, c->st.pos + pair * B, B * 4, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess && score_host)
+    e = cudaMemcpyAsync(score_host, c->st.score + pair * B, B * 4, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess && nvalid_host)
+    e = cudaMemcpyAsync(nvalid_host, c->st.nvalid + pair, 4, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  return poison_on(c, e);
+}
+
+}  // extern "C"

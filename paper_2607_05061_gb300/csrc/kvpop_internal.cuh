@@ -1,0 +1,101 @@
+// Internal declarations shared by the KVpop CUDA translation units.
+// Not part of the public ABI (see include/kvpop.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/kvpop.h"
+
+namespace kvpop {
+
+typedef __nv_bfloat16 bf16;
+
+// Device-side error codes written to cache->err[0] (first error wins).
+enum : int {
+  DEVERR_NONE = 0,
+  DEVERR_TIMEOUT_FULL = 1,     // consumer gave up waiting for a K/V tile
+  DEVERR_TIMEOUT_EMPTY = 2,    // producer gave up waiting for a free stage
+  DEVERR_TIMEOUT_DRAIN = 3,    // producer gave up draining its copies at exit
+  DEVERR_BAD_SCHEDULE = 4,     // attention schedule inconsistent with the state
+};
+
+// Wall-clock budget of any single mbarrier wait before a kernel gives up.
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+struct State {                 // device pointers of one cache
+  void* slotK;                 // [pairs][B][d]   element type T
+  void* slotV;
+  void* ringK;                 // [pairs][D][d]
+  void* ringV;
+  float* ringQm;               // [pairs][D][d]   mean query of each window token
+  float* score;                // [pairs][B]      static priority of each slot
+  int32_t* pos;                // [pairs][B]      position held by each slot
+  int32_t* nvalid;             // [pairs]
+  int32_t* len;                // [pairs]         tokens seen (same for all heads of a sequence)
+  float* min_score;            // [pairs]         argmin over slots [s, B) when full
+  int32_t* min_slot;           // [pairs]
+  // scorer
+  const float* W1;             // [H][3d][F]
+  const float* b1;             // [H][F]
+  const float* w2;             // [H][F]
+  const float* b2;             // [H]
+  const float* log_gamma;      // [H] or nullptr
+  // attention workspace
+  float* part;                 // [2 * grid][G*d + 2*G]
+  int32_t* part_count;         // [pairs]
+  int32_t* err;                // [4]
+};
+
+struct Dims {
+  int batch, H, G, d, B, D, s, F;
+  int dtype;                   // kvpop_dtype
+  int pairs;
+};
+
+// ------------------------------------------------------------------ launchers
+cudaError_t launch_ingest(const State& st, const Dims& dm, const void* q, const void* k,
+                          const void* v, const float* override_, int32_t* evict_info,
+                          float* score_out, cudaStream_t stream);
+
+// Attention kernel resources for a (dtype, d, G) combination.
+struct AttendConfig {
+  int threads;
+  size_t smem_fixed;           // bytes independent of the number of pairs
+  int tile;                    // keys per tile
+  const void* func;            // kernel symbol (for occupancy queries)
+};
+cudaError_t attend_config(const Dims& dm, AttendConfig* out);
+cudaError_t launch_attend(const State& st, const Dims& dm, const void* q, float* out,
+                          int grid, cudaStream_t stream);
+
+cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const void* K,
+                           const void* V, const int32_t* plen_dev, int first_seq, int n_seq,
+                           int Pmax, const float* override_, float* tmp_prio,
+                           cudaStream_t stream);
+
+// ------------------------------------------------------------------ device helpers
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+
+// Canonical score: NaN -> -inf, -0 -> +0 (every ranking decision uses it).
+__device__ __forceinline__ float canon_score(float r) {
+  if (r != r) return -INFINITY;
+  return r + 0.0f;   // -0 + +0 = +0 under round-to-nearest
+}
+
+// Static priority (App. B.3, decay step n = 1) in explicit fp32 ops.
+__device__ __forceinline__ float static_priority(float r, int u, const float* log_gamma, int h) {
+  if (log_gamma == nullptr) return r;
+  float lg = log_gamma[h];
+  if (lg == 0.0f) return r;
+  return canon_score(__fsub_rn(r, __fmul_rn((float)u, lg)));
+}
+
+// Exact-erf GELU.
+__device__ __forceinline__ float gelu_erf(float z) {
+  return 0.5f * z * (1.0f + erff(z * 0.70710678118654752440f));
+}
+
+}  // namespace kvpop

@@ -1,0 +1,200 @@
+"""ctypes binding of the KVpop C ABI (include/kvpop.h).
+
+Argument marshalling only: every step of the decode path runs in the CUDA
+library ``libkvpop.so``.  Tensors are passed by ``data_ptr()`` and the current
+torch stream by its ``cuda_stream`` handle; torch is used only for device
+memory and streams.  Importing this module fails loudly when the library has
+not been built -- there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int32, c_size_t, c_void_p
+from typing import Optional, Sequence
+
+import torch  # loads the CUDA runtime the library links against
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libkvpop.so")
+
+KVPOP_F32, KVPOP_BF16 = 0, 1
+STATUS = {0: "KVPOP_OK", 1: "KVPOP_ERR_INVALID_ARG", 2: "KVPOP_ERR_ALIGN", 3: "KVPOP_ERR_OOM",
+          4: "KVPOP_ERR_CUDA", 5: "KVPOP_ERR_STATE", 6: "KVPOP_ERR_DEVICE_CHECK"}
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_05061_gb300.build`"
+                      " (or __graft_entry__.build()); the decode path has no non-CUDA fallback")
+_lib = ctypes.CDLL(LIB_PATH)
+
+
+class kvpop_config(ctypes.Structure):
+    _fields_ = [("batch", c_int32), ("n_kv_heads", c_int32), ("q_per_kv", c_int32),
+                ("head_dim", c_int32), ("budget_B", c_int32), ("delay_D", c_int32),
+                ("n_sink", c_int32), ("scorer_hidden", c_int32), ("kv_dtype", ctypes.c_int)]
+
+
+class kvpop_scorer(ctypes.Structure):
+    _fields_ = [("W1", c_void_p), ("b1", c_void_p), ("w2", c_void_p), ("b2", c_void_p),
+                ("log_gamma", c_void_p)]
+
+
+_P = c_void_p
+_SIGS = {
+    "kvpop_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "kvpop_init_cache": (ctypes.c_int, [POINTER(kvpop_config), POINTER(kvpop_scorer), _P, POINTER(_P)]),
+    "kvpop_free": (ctypes.c_int, [_P]),
+    "kvpop_prefill_compress": (ctypes.c_int, [_P, _P, _P, _P, POINTER(c_int32), c_int32, c_int32,
+                                              c_int32, _P, _P]),
+    "kvpop_decode_ingest": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P]),
+    "kvpop_decode_attend": (ctypes.c_int, [_P, _P, _P, _P]),
+    "kvpop_decode_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P]),
+    "kvpop_decode_step_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P]),
+    "kvpop_check": (ctypes.c_int, [_P, _P]),
+    "kvpop_export_state": (ctypes.c_int, [_P, _P, POINTER(c_size_t), _P]),
+    "kvpop_import_state": (ctypes.c_int, [_P, _P, c_size_t, _P]),
+    "kvpop_get_lengths": (ctypes.c_int, [_P, POINTER(c_int32), _P]),
+    "kvpop_get_pair_state": (ctypes.c_int, [_P, c_int32, c_int32, POINTER(c_int32), POINTER(c_float),
+                                            POINTER(c_int32), _P]),
+    "kvpop_debug_fail_alloc_after": (None, [c_int32]),
+}
+for _name, (_res, _args) in _SIGS.items():
+    _fn = getattr(_lib, _name)
+    _fn.restype = _res
+    _fn.argtypes = _args
+    globals()[_name] = _fn
+
+EXPORTED = tuple(_SIGS)
+
+
+class KVpopError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        msg = kvpop_status_string(status).decode()
+        super().__init__(f"{what}: {STATUS.get(status, status)} ({msg})")
+
+
+def _ck(status: int, what: str):
+    if status != 0:
+        raise KVpopError(status, what)
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream=None) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def dtype_code(dtype) -> int:
+    return KVPOP_F32 if dtype in ("f32", torch.float32) else KVPOP_BF16
+
+
+class KVpopCache:
+    """One attention layer's compressed KV cache (library-owned device state)."""
+
+    def __init__(self, batch: int, n_kv_heads: int, q_per_kv: int, head_dim: int, budget_B: int,
+                 delay_D: int, scorer_hidden: int, kv_dtype, W1, b1, w2, b2, log_gamma=None,
+                 n_sink: int = 0, stream=None):
+        self.cfg = kvpop_config(batch, n_kv_heads, q_per_kv, head_dim, budget_B, delay_D, n_sink,
+                                scorer_hidden, dtype_code(kv_dtype))
+        keep = [t.contiguous().float() for t in (W1, b1, w2, b2)]
+        lg = None if log_gamma is None else log_gamma.contiguous().float()
+        sc = kvpop_scorer(*[t.data_ptr() for t in keep], None if lg is None else lg.data_ptr())
+        h = _P()
+        _ck(kvpop_init_cache(ctypes.byref(self.cfg), ctypes.byref(sc), _stream(stream), ctypes.byref(h)),
+            "kvpop_init_cache")
+        self.handle = h.value
+        self.batch, self.H, self.G, self.d = batch, n_kv_heads, q_per_kv, head_dim
+
+    def prefill(self, Q, K, V, prompt_lens: Sequence[int], first_seq: int = 0, override=None,
+                stream=None):
+        n_seq = len(prompt_lens)
+        arr = (c_int32 * n_seq)(*[int(x) for x in prompt_lens])
+        Pmax = K.shape[2] if K is not None else 0
+        _ck(kvpop_prefill_compress(self.handle, _ptr(Q), _ptr(K), _ptr(V), arr, first_seq, n_seq, Pmax,
+                                   _ptr(override), _stream(stream)), "kvpop_prefill_compress")
+
+    def ingest(self, q, k, v, override=None, evict_info=None, score_out=None, stream=None):
+        _ck(kvpop_decode_ingest(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(override),
+                                _ptr(evict_info), _ptr(score_out), _stream(stream)), "kvpop_decode_ingest")
+
+    def attend(self, q, out, stream=None):
+        _ck(kvpop_decode_attend(self.handle, _ptr(q), _ptr(out), _stream(stream)), "kvpop_decode_attend")
+
+    def step(self, q, k, v, out, override=None, evict_info=None, score_out=None, stream=None):
+        _ck(kvpop_decode_step(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(override),
+                              _ptr(evict_info), _ptr(score_out), _stream(stream)), "kvpop_decode_step")
+
+    def step_host(self, q, k, v, out, stream=None):
+        _ck(kvpop_decode_step_host(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), _stream(stream)),
+            "kvpop_decode_step_host")
+
+    def check(self, stream=None):
+        _ck(kvpop_check(self.handle, _stream(stream)), "kvpop_check")
+
+    def lengths(self, stream=None):
+        arr = (c_int32 * self.batch)()
+        _ck(kvpop_get_lengths(self.handle, arr, _stream(stream)), "kvpop_get_lengths")
+        return list(arr)
+
+    def pair_state(self, seq: int, head: int, stream=None):
+        """(positions of the used slots in slot order, their priorities) of one KV head."""
+        B = self.cfg.budget_B
+        pos = (c_int32 * B)()
+        sc = (c_float * B)()
+        nv = c_int32(0)
+        _ck(kvpop_get_pair_state(self.handle, seq, head, pos, sc, ctypes.byref(nv), _stream(stream)),
+            "kvpop_get_pair_state")
+        n = nv.value
+        return list(pos)[:n], list(sc)[:n]
+
+    def export_state(self, stream=None) -> bytes:
+        n = c_size_t(0)
+        _ck(kvpop_export_state(self.handle, None, ctypes.byref(n), _stream(stream)), "kvpop_export_state")
+        buf = ctypes.create_string_buffer(n.value)
+        _ck(kvpop_export_state(self.handle, buf, ctypes.byref(n), _stream(stream)), "kvpop_export_state")
+        return buf.raw
+
+    def import_state(self, blob: bytes, stream=None):
+        _ck(kvpop_import_state(self.handle, blob, len(blob), _stream(stream)), "kvpop_import_state")
+
+    def free(self):
+        if getattr(self, "handle", None):
+            _ck(kvpop_free(self.handle), "kvpop_free")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def parse_state(blob: bytes, cfg: kvpop_config) -> dict:
+    """Split a ``kvpop_export_state`` blob into named numpy arrays (checkpoint inspection)."""
+    import numpy as np
+    pairs = cfg.batch * cfg.n_kv_heads
+    B, D, d = cfg.budget_B, cfg.delay_D, cfg.head_dim
+    kv_np = np.float32 if cfg.kv_dtype == KVPOP_F32 else np.uint16   # bf16 kept as raw bits
+    esz = 4 if cfg.kv_dtype == KVPOP_F32 else 2
+    layout = [("slotK", kv_np, (pairs, B, d), esz), ("slotV", kv_np, (pairs, B, d), esz),
+              ("ringK", kv_np, (pairs, D, d), esz), ("ringV", kv_np, (pairs, D, d), esz),
+              ("ringQm", np.float32, (pairs, D, d), 4), ("score", np.float32, (pairs, B), 4),
+              ("pos", np.int32, (pairs, B), 4), ("nvalid", np.int32, (pairs,), 4),
+              ("len", np.int32, (pairs,), 4), ("min_score", np.float32, (pairs,), 4),
+              ("min_slot", np.int32, (pairs,), 4)]
+    off = 4 * 8 + ctypes.sizeof(kvpop_config)
+    out = {}
+    for name, dt, shape, sz in layout:
+        n = int(np.prod(shape)) * sz
+        out[name] = np.frombuffer(blob, dtype=dt, count=int(np.prod(shape)), offset=off).reshape(shape)
+        off += n
+    return out

@@ -1,0 +1,263 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the
+same seeded inputs.
+
+* Evictions (slot, evicted position) must match bit for bit when both sides
+  consume the same scores (the oracle's own fp32 scores, or injected ones).
+* Attention outputs must match within max-abs 1e-5 (fp32 K/V) or 2e-2 (bf16).
+* The GPU scorer is compared with the oracle's scorer value by value, and the
+  end-to-end eviction agreement with the GPU's own scores is reported.
+"""
+import numpy as np
+import pytest
+import torch
+
+from gpu_harness import (TOL, compare, gpu_decode, gpu_prefill, injected_decode_scores,
+                         injected_prefill_scores, make_cache, oracle_pairs)
+from workload import gen, get_config
+
+pytestmark = pytest.mark.gpu
+
+
+def all_pairs(cfg):
+    return [(b, h) for b in range(cfg.batch) for h in range(cfg.n_kv_heads)]
+
+
+# ---------------------------------------------------------------- tiny config, full
+def test_tiny_bitexact_with_oracle_scores(cuda_device):
+    cfg = get_config("tiny")
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    steps = cfg.decode_steps
+    ref = oracle_pairs(cfg, w, L, steps, pairs)             # oracle with its own scorer
+    Pmax = max(L)
+    pov = torch.zeros((cfg.batch, cfg.n_kv_heads, Pmax), dtype=torch.float32)
+    dov = torch.zeros((steps, cfg.batch, cfg.n_kv_heads), dtype=torch.float32)
+    for (b, h), tr in zip(pairs, ref):
+        raw = tr.cache.prefill_raw
+        pov[b, h, :raw.size] = torch.from_numpy(raw)
+        dov[:, b, h] = torch.tensor(np.asarray(tr.scores, dtype=np.float32))
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    pre = oracle_pairs(cfg, w, L, 0, pairs, prefill_override=pov)
+    for (b, h), t in zip(pairs, pre):
+        pos, _ = cache.pair_state(b, h)
+        assert pos == t.cache.kept_positions()
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device))
+    err = compare(cfg, g, ref, pairs)
+    print(f"tiny: max-abs attention error {err:.3e} over {steps} steps")
+    assert err <= TOL["f32"]
+    cache.free()
+
+
+def test_tiny_gpu_scorer_against_oracle(cuda_device):
+    cfg = get_config("tiny")
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    steps = cfg.decode_steps
+    ref = oracle_pairs(cfg, w, L, steps, pairs)
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device)
+    # prefill: kept set agreement and per-slot priorities of the common slots
+    agree = []
+    for (b, h), tr in zip(pairs, ref):
+        pos, sc = cache.pair_state(b, h)
+        o = set(tr.cache.kept_positions())
+        agree.append(len(o & set(pos)) / max(1, len(o)))
+        raw = tr.cache.prefill_raw
+        for p_, s_ in zip(pos, sc):
+            assert abs(s_ - float(raw[p_])) <= 2e-5 * (1.0 + abs(float(raw[p_])))
+    g = gpu_decode(cache, cfg, L, steps, cuda_device)
+    n_same, n_all = 0, 0
+    for (b, h), tr in zip(pairs, ref):
+        want = np.asarray(tr.scores, dtype=np.float64)
+        got = g.scores[:, b, h].astype(np.float64)
+        assert np.all(np.abs(got - want) <= 2e-5 * (1.0 + np.abs(want))), "scorer mismatch"
+        ev = g.evict[:, b, h]
+        n_same += int(((ev[:, 0] == np.asarray(tr.slots)) & (ev[:, 1] == np.asarray(tr.evicted))).sum())
+        n_all += steps
+    print(f"tiny: prefill kept-set agreement {np.mean(agree):.4f}; "
+          f"decode eviction agreement with GPU scores {n_same / n_all:.4f}")
+    cache.free()
+
+
+# ---------------------------------------------------------------- reduced bf16, all pairs
+SMALL = dict(batch=2, prompt_len=600, budget_B=256, decode_steps=200)
+
+
+@pytest.mark.parametrize("name,over", [
+    ("q4b", SMALL),
+    ("q4b", dict(SMALL, n_sink=3)),
+    ("q4b", dict(SMALL, log_gamma=-0.002)),
+    ("q4b", dict(SMALL, budget_B=1, delay_D=1, prompt_len=40, decode_steps=60)),
+    ("q4b", dict(SMALL, budget_B=900, prompt_len=300, decode_steps=100)),       # B >= context: dense
+    ("q4b", dict(SMALL, prompt_len=5, decode_steps=80)),                       # P < D
+    ("q4b", dict(SMALL, prompt_len=0, decode_steps=70)),                       # no prompt
+    ("q4b", dict(SMALL, q_per_kv=1, head_dim=64)),
+    ("q4b", dict(SMALL, q_per_kv=2)),
+    ("tiny", dict(batch=3, head_dim=128, q_per_kv=4, prompt_len=200, budget_B=40, delay_D=7,
+                  decode_steps=120)),
+    ("tiny", dict(q_per_kv=1, prompt_len=90, budget_B=16, delay_D=2, decode_steps=90)),
+])
+def test_injected_scores_bitexact(cuda_device, name, over):
+    cfg = get_config(name, **over)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    steps = cfg.decode_steps
+    Pmax = max(1, max(L))
+    pov = injected_prefill_scores(cfg, Pmax, "cpu")
+    dov = injected_decode_scores(cfg, steps, "cpu")
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device))
+    ref = oracle_pairs(cfg, w, L, steps, pairs, prefill_override=pov, decode_override=dov)
+    err = compare(cfg, g, ref, pairs)
+    print(f"{name} {over}: max-abs attention error {err:.3e}")
+    assert err <= TOL[cfg.kv_dtype]
+    cache.free()
+
+
+def test_planted_ties_bitexact(cuda_device):
+    """Scores drawn from 3 levels: argmin ties (lowest slot) and strict-beat drops."""
+    cfg = get_config("q4b", batch=2, prompt_len=300, budget_B=64, decode_steps=150)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    pov = injected_prefill_scores(cfg, max(L), "cpu", levels=3)
+    dov = injected_decode_scores(cfg, cfg.decode_steps, "cpu", levels=3)
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    g = gpu_decode(cache, cfg, L, cfg.decode_steps, cuda_device, override=dov.to(cuda_device))
+    ref = oracle_pairs(cfg, w, L, cfg.decode_steps, pairs, prefill_override=pov, decode_override=dov)
+    assert compare(cfg, g, ref, pairs) <= TOL["bf16"]
+    cache.free()
+
+
+# ---------------------------------------------------------------- full sizes, sampled pairs
+@pytest.mark.parametrize("name,steps,sample", [
+    ("q4b", 256, [(0, 0), (3, 5), (7, 7)]),
+    ("cr8x", 48, [(0, 0), (63, 7)]),
+    ("ragged", 24, None),
+])
+def test_full_size_sampled(cuda_device, name, steps, sample):
+    cfg = get_config(name)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    if sample is None:   # shortest and longest sequence, and one below the budget
+        order = sorted(range(cfg.batch), key=lambda b: L[b])
+        below = [b for b in order if L[b] - cfg.delay_D < cfg.budget_B]
+        sample = [(order[0], 1), (order[-1], 6)] + ([(below[-1], 3)] if below else [])
+    Pmax = max(L)
+    pov = injected_prefill_scores(cfg, Pmax, cuda_device)
+    dov = injected_decode_scores(cfg, steps, cuda_device)
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov)
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov, sample=sample)
+    ref = oracle_pairs(cfg, w, L, steps, sample, prefill_override=pov.cpu(),
+                       decode_override=dov.cpu())
+    err = 0.0
+    for i, ((b, h), tr) in enumerate(zip(sample, ref)):
+        pos, _ = cache.pair_state(b, h)
+        assert len(pos) == min(cfg.budget_B, max(0, L[b] + steps - cfg.delay_D))
+        sub = type(g)(g.evict, g.scores, g.outputs[:, i:i + 1])
+        err = max(err, compare(cfg, sub, [tr], [(b, h)]))
+    print(f"{name}: sampled max-abs attention error {err:.3e}")
+    assert err <= TOL[cfg.kv_dtype]
+    cache.free()
+
+
+def test_full_size_gpu_scorer(cuda_device):
+    """cr8x shape, GPU scorer: per-token scores vs the oracle scorer on sampled pairs."""
+    cfg = get_config("cr8x", batch=8)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    steps = 32
+    sample = [(0, 0), (5, 3)]
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device)
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, sample=sample)
+    ref = oracle_pairs(cfg, w, L, steps, sample, attend=False)
+    for (b, h), tr in zip(sample, ref):
+        want = np.asarray(tr.scores, dtype=np.float64)
+        got = g.scores[:, b, h].astype(np.float64)
+        assert np.all(np.abs(got - want) <= 5e-5 * (1.0 + np.abs(want)))
+        pos, sc = cache.pair_state(b, h)
+        o = set(tr.cache.kept_positions())
+        print(f"cr8x GPU scorer {(b, h)}: final kept-set agreement "
+              f"{len(o & set(pos)) / len(o):.4f}")
+    cache.free()
+
+
+# ---------------------------------------------------------------- API behaviour
+def test_checkpoint_resume_is_bit_identical(cuda_device):
+    cfg = get_config("q4b", batch=2, prompt_len=500, budget_B=128, decode_steps=60)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    a = make_cache(cfg, w)
+    gpu_prefill(a, cfg, L, cuda_device)
+    gpu_decode(a, cfg, L, 30, cuda_device)
+    blob = a.export_state()
+    b = make_cache(cfg, w)
+    b.import_state(blob)
+    ga = gpu_decode(a, cfg, L, 30, cuda_device, step0=30)
+    gb = gpu_decode(b, cfg, L, 30, cuda_device, step0=30)
+    assert np.array_equal(ga.evict, gb.evict)
+    assert np.array_equal(ga.outputs, gb.outputs)
+    assert a.lengths() == [x + 60 for x in L]
+    a.free()
+    b.free()
+
+
+def test_host_buffer_step_matches_device_step(cuda_device):
+    cfg = get_config("q4b", batch=2, prompt_len=300, budget_B=64, decode_steps=20)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    a, b = make_cache(cfg, w), make_cache(cfg, w)
+    gpu_prefill(a, cfg, L, cuda_device)
+    gpu_prefill(b, cfg, L, cuda_device)
+    q, k, v = gen.decode_inputs(cfg, L, 0, 20, device="cpu")
+    out_d = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), device=cuda_device)
+    out_h = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim)).pin_memory()
+    for j in range(20):
+        a.step(q[j].to(cuda_device), k[j].to(cuda_device), v[j].to(cuda_device), out_d)
+        b.step_host(q[j].pin_memory(), k[j].pin_memory(), v[j].pin_memory(), out_h)
+        torch.cuda.synchronize()
+        assert torch.equal(out_d.cpu(), out_h)
+    a.free()
+    b.free()
+
+
+def test_alloc_failure_is_reported_and_recoverable(cuda_device):
+    from paper_2607_05061_gb300 import kvpop
+    cfg = get_config("tiny")
+    w = gen.scorer_weights(cfg)
+    for n in (1, 3, 7, 12):
+        kvpop.kvpop_debug_fail_alloc_after(n)
+        with pytest.raises(kvpop.KVpopError) as ei:
+            make_cache(cfg, w)
+        assert ei.value.status == 3
+    kvpop.kvpop_debug_fail_alloc_after(0)
+    c = make_cache(cfg, w)
+    c.check()
+    c.free()
+
+
+def test_misaligned_and_bad_arguments(cuda_device):
+    from paper_2607_05061_gb300 import kvpop
+    cfg = get_config("q4b", batch=1, prompt_len=64, budget_B=32)
+    c = make_cache(cfg, gen.scorer_weights(cfg))
+    buf = torch.zeros(4096, dtype=torch.bfloat16, device=cuda_device)
+    out = torch.zeros(4096, dtype=torch.float32, device=cuda_device)
+    with pytest.raises(kvpop.KVpopError) as ei:
+        c.ingest(buf.data_ptr() + 2, buf, buf)
+    assert ei.value.status == 2
+    with pytest.raises(kvpop.KVpopError) as ei:
+        c.attend(buf, out.data_ptr() + 4)
+    assert ei.value.status == 2
+    with pytest.raises(kvpop.KVpopError) as ei:
+        c.prefill(buf, buf, buf, [10, 10])          # two sequences in a batch of one
+    assert ei.value.status == 1
+    c.check()
+    c.free()
