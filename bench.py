@@ -40,6 +40,10 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["kvpop", "reference"], default="kvpop")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch (small profiling cases)")
+    ap.add_argument("--prompt-len", type=int, default=None,
+                    help="override the workload's prompt length (small profiling cases)")
     ap.add_argument("--e2e-steps", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=96)
@@ -226,7 +230,12 @@ def run_kvpop(args):
     from paper_2607_05061_gb300 import kvpop
     from workload import gen, get_config
 
-    cfg = get_config(args.config)
+    over = {}
+    if args.batch:
+        over["batch"] = args.batch
+    if args.prompt_len:
+        over["prompt_len"] = args.prompt_len
+    cfg = get_config(args.config, **over)
     if cfg.n_layers != 1:
         raise SystemExit("bench.py times single-layer workloads (tiny, q4b, cr8x, ragged)")
     L = gen.prompt_lengths(cfg)

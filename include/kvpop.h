@@ -23,7 +23,9 @@
  *
  * Conventions for every call:
  *  - Pointers named *_dev are device pointers; *_host are host pointers.
- *    Device pointers must be 16-byte aligned, else KVPOP_ERR_ALIGN.
+ *    q/k/v/Q/K/V/out device pointers must be 16-byte aligned and the small
+ *    per-(sequence, head) arrays (score overrides, evict_info, score_out)
+ *    4-byte aligned, else KVPOP_ERR_ALIGN.
  *  - Calls are asynchronous on `stream` unless stated; the caller owns every
  *    input/output buffer, the library owns the cache.
  *  - No call aborts or throws; each returns a status.  After a CUDA error the
@@ -165,6 +167,10 @@ kvpop_status kvpop_get_lengths(kvpop_cache* cache, int32_t* len_host, cudaStream
 kvpop_status kvpop_get_pair_state(kvpop_cache* cache, int32_t seq, int32_t head,
                                   int32_t* pos_host, float* score_host, int32_t* nvalid_host,
                                   cudaStream_t stream);
+
+/* Description of the last failing CUDA call made by this library on the
+ * calling thread ("" if none): call site, error name and message. */
+const char* kvpop_last_error(void);
 
 /* Testing hook: make the n-th device allocation from now fail (n >= 1), or
  * disable with n <= 0.  Affects only this library's allocations. */

@@ -16,7 +16,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkvpop.so")
-SOURCES = ["kvpop_api.cu", "kvpop_ingest.cu", "kvpop_attend.cu", "kvpop_prefill.cu"]
+SOURCES = ["kvpop_api.cu", "kvpop_ingest.cu", "kvpop_attend.cu", "kvpop_attend_tc.cu",
+           "kvpop_prefill.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -49,8 +50,8 @@ def _compile(src: str, verbose_ptxas: bool) -> str:
 
 def build(verbose_ptxas: bool = False, force: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
-    srcs = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "kvpop_internal.cuh"),
-                                                     os.path.join(HERE, "..", "include", "kvpop.h")]
+    srcs = ([os.path.join(CSRC, s) for s in os.listdir(CSRC)]
+            + [os.path.join(HERE, "..", "include", "kvpop.h")])
     if (not force and os.path.exists(LIB)
             and os.path.getmtime(LIB) > max(os.path.getmtime(s) for s in srcs)):
         return LIB

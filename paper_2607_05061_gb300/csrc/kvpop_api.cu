@@ -5,7 +5,7 @@
 #include <new>
 #include <vector>
 
-#include "kvpop_internal.cuh"
+#include "kvpop_argmin.cuh"
 
 using namespace kvpop;
 
@@ -24,6 +24,8 @@ struct kvpop_cache {
   bool poisoned = false;
   bool has_decay = false;
   std::vector<void*> allocs;
+  std::vector<unsigned char> tc_maps;   // TMA descriptors of the K/V stores (bf16 path)
+  bool use_tc = false;
   // staging for kvpop_decode_step_host
   void* stage_q = nullptr;
   void* stage_k = nullptr;
@@ -37,6 +39,16 @@ namespace {
 constexpr uint64_t kMagic = 0x6b7670'6f70'6361ull;   // "kvpopca"
 constexpr uint64_t kStateVersion = 1;
 int g_fail_after = 0;
+thread_local char g_last_error[256] = "";
+
+// Record the failing call (file-local line) for kvpop_last_error().
+cudaError_t note(cudaError_t e, int line) {
+  if (e != cudaSuccess)
+    std::snprintf(g_last_error, sizeof(g_last_error), "kvpop_api.cu:%d: %s (%s)", line,
+                  cudaGetErrorName(e), cudaGetErrorString(e));
+  return e;
+}
+#define NOTE(expr) note((expr), __LINE__)
 
 kvpop_status from_cuda(cudaError_t e) {
   if (e == cudaSuccess) return KVPOP_OK;
@@ -45,12 +57,13 @@ kvpop_status from_cuda(cudaError_t e) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
 kvpop_status dev_alloc(kvpop_cache* c, void** p, size_t bytes) {
   *p = nullptr;
   if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
   if (bytes == 0) bytes = 16;
-  cudaError_t e = cudaMalloc(p, bytes);
+  cudaError_t e = NOTE(cudaMalloc(p, bytes));
   if (e != cudaSuccess) {
     cudaGetLastError();   // clear the sticky-free allocation error
     *p = nullptr;
@@ -63,6 +76,12 @@ kvpop_status dev_alloc(kvpop_cache* c, void** p, size_t bytes) {
 void release(kvpop_cache* c) {
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
+}
+
+// 64-byte aligned view of the stored TMA descriptors.
+void* tc_map_ptr(kvpop_cache* c) {
+  uintptr_t p = reinterpret_cast<uintptr_t>(c->tc_maps.data());
+  return reinterpret_cast<void*>((p + 63) & ~uintptr_t(63));
 }
 
 kvpop_status validate(const kvpop_config* cfg) {
@@ -112,6 +131,8 @@ std::vector<StateBuf> state_buffers(kvpop_cache* c) {
       {c->st.len, pairs * 4},
       {c->st.min_score, pairs * 4},
       {c->st.min_slot, pairs * 4},
+      {c->st.blk_score, pairs * min_blocks(dm.B) * 4},
+      {c->st.blk_slot, pairs * min_blocks(dm.B) * 4},
   };
 }
 
@@ -134,6 +155,8 @@ const char* kvpop_status_string(kvpop_status s) {
 
 void kvpop_debug_fail_alloc_after(int32_t n) { g_fail_after = n > 0 ? n : 0; }
 
+const char* kvpop_last_error(void) { return g_last_error; }
+
 kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
                               cudaStream_t stream, kvpop_cache** out) {
   if (!out) return KVPOP_ERR_INVALID_ARG;
@@ -148,16 +171,19 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
   Dims& dm = c->dm;
   dm.batch = cfg->batch; dm.H = cfg->n_kv_heads; dm.G = cfg->q_per_kv; dm.d = cfg->head_dim;
   dm.B = cfg->budget_B; dm.D = cfg->delay_D; dm.s = cfg->n_sink; dm.F = cfg->scorer_hidden;
+  dm.Fp = (dm.F + 3) & ~3;
   dm.dtype = cfg->kv_dtype;
   dm.pairs = dm.batch * dm.H;
   c->esz = cfg->kv_dtype == KVPOP_F32 ? 4 : 2;
   c->magic = kMagic;
-  cudaGetDevice(&c->device);
+  NOTE(cudaGetDevice(&c->device));
 
-  const size_t pairs = dm.pairs, B = dm.B, D = dm.D, d = dm.d, H = dm.H, F = dm.F;
+  const size_t pairs = dm.pairs, B = dm.B, D = dm.D, d = dm.d, H = dm.H, F = dm.F, Fp = dm.Fp;
+  const size_t NB = min_blocks(dm.B);
   const size_t I = 3 * d;
   AttendConfig ac;
-  kvpop_status s = from_cuda(attend_config(dm, &ac));
+  c->use_tc = cfg->kv_dtype == KVPOP_BF16;
+  kvpop_status s = from_cuda(NOTE(c->use_tc ? tc_config(dm, &ac) : attend_config(dm, &ac)));
   void* p = nullptr;
 #define ALLOC(field, type, bytes)                        \
   if (s == KVPOP_OK) {                                   \
@@ -175,18 +201,21 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
   ALLOC(len, int32_t*, pairs * 4)
   ALLOC(min_score, float*, pairs * 4)
   ALLOC(min_slot, int32_t*, pairs * 4)
+  ALLOC(blk_score, float*, pairs * NB * 4)
+  ALLOC(blk_slot, int32_t*, pairs * NB * 4)
   float* w = nullptr;
-  if (s == KVPOP_OK) { s = dev_alloc(c, &p, (H * I * F + 2 * H * F + 2 * H) * 4); w = (float*)p; }
+  const size_t wbytes = (H * I * Fp + 2 * H * Fp + 2 * H) * 4;
+  if (s == KVPOP_OK) { s = dev_alloc(c, &p, wbytes); w = (float*)p; }
   ALLOC(part_count, int32_t*, pairs * 4)
-  ALLOC(err, int32_t*, 16)
+  ALLOC(err, int32_t*, 16 * 4)
   int sms = 0, occ = 0;
   if (s == KVPOP_OK) {
-    s = from_cuda(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
+    s = from_cuda(NOTE(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device)));
     const size_t smem = ac.smem_fixed + (pairs + 1) * 4;
     if (s == KVPOP_OK)
-      s = from_cuda(cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+      s = from_cuda(NOTE(cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)));
     if (s == KVPOP_OK)
-      s = from_cuda(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ac.func, ac.threads, smem));
+      s = from_cuda(NOTE(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ac.func, ac.threads, smem)));
     if (s == KVPOP_OK && occ < 1) s = KVPOP_ERR_INVALID_ARG;
     c->attend_grid = sms * (occ > 0 ? occ : 1);
   }
@@ -196,32 +225,47 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
   if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_k = p; }
   if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_v = p; }
   if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * 4); c->stage_out = (float*)p; }
-  if (s == KVPOP_OK) s = from_cuda(prepare_ingest(dm));
-  if (s == KVPOP_OK) s = from_cuda(prepare_prefill(dm));
+  if (s == KVPOP_OK && c->use_tc) {
+    c->tc_maps.assign(tc_maps_size() + 64, 0);
+    s = from_cuda(NOTE(tc_make_maps(c->st, dm, tc_map_ptr(c))));
+  }
+  if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest(dm)));
+  if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_prefill(dm)));
   if (s == KVPOP_OK) {
     float* W1 = w;
-    float* b1 = W1 + H * I * F;
-    float* w2 = b1 + H * F;
-    float* b2 = w2 + H * F;
+    float* b1 = W1 + H * I * Fp;
+    float* w2 = b1 + H * Fp;
+    float* b2 = w2 + H * Fp;
     float* lg = b2 + H;
     c->st.W1 = W1; c->st.b1 = b1; c->st.w2 = w2; c->st.b2 = b2;
-    cudaError_t e = cudaMemcpyAsync(W1, sc->W1, H * I * F * 4, cudaMemcpyDefault, stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(b1, sc->b1, H * F * 4, cudaMemcpyDefault, stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(w2, sc->w2, H * F * 4, cudaMemcpyDefault, stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream);
+    // hidden units padded to Fp with zero weights: rows of F floats into rows of Fp
+    cudaError_t e = NOTE(cudaMemsetAsync(w, 0, wbytes, stream));
+    if (e == cudaSuccess)
+      e = NOTE(cudaMemcpy2DAsync(W1, Fp * 4, sc->W1, F * 4, F * 4, H * I, cudaMemcpyDefault, stream));
+    if (e == cudaSuccess)
+      e = NOTE(cudaMemcpy2DAsync(b1, Fp * 4, sc->b1, F * 4, F * 4, H, cudaMemcpyDefault, stream));
+    if (e == cudaSuccess)
+      e = NOTE(cudaMemcpy2DAsync(w2, Fp * 4, sc->w2, F * 4, F * 4, H, cudaMemcpyDefault, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && sc->log_gamma) {
-      e = cudaMemcpyAsync(lg, sc->log_gamma, H * 4, cudaMemcpyDefault, stream);
+      e = NOTE(cudaMemcpyAsync(lg, sc->log_gamma, H * 4, cudaMemcpyDefault, stream));
       c->st.log_gamma = lg;
       c->has_decay = true;
     } else {
       c->st.log_gamma = nullptr;
     }
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.nvalid, 0, pairs * 4, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.len, 0, pairs * 4, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.part_count, 0, pairs * 4, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.err, 0, 16 * 4, stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->st.pos, 0xff, pairs * B * 4, stream);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.nvalid, 0, pairs * 4, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.len, 0, pairs * 4, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.part_count, 0, pairs * 4, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.err, 0, 16 * 4, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.pos, 0xff, pairs * B * 4, stream));
+    // zeroed K/V stores: rows past the used slots are read (with weight 0) by the
+    // tensor-core attention tiles and must hold finite values
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.slotK, 0, pairs * B * d * c->esz, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.slotV, 0, pairs * B * d * c->esz, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.ringK, 0, pairs * D * d * c->esz, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.ringV, 0, pairs * D * d * c->esz, stream));
+    if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
     s = from_cuda(e);
   }
   if (s != KVPOP_OK) {
@@ -257,24 +301,24 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
   for (int i = 0; i < n_seq; ++i)
     if (plen_host[i] < 0 || plen_host[i] > Pmax) return KVPOP_ERR_INVALID_ARG;
   if (Pmax > 0 && (!Q || !K || !V)) return KVPOP_ERR_INVALID_ARG;
-  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(override_))
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned4(override_))
     return KVPOP_ERR_ALIGN;
   const size_t pairs = (size_t)n_seq * c->dm.H;
   const size_t prio_bytes = pairs * (size_t)Pmax * 4;
   void* tmp = nullptr;
   if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
-  cudaError_t e = cudaMallocAsync(&tmp, prio_bytes + 256 + (size_t)n_seq * 4, stream);
+  cudaError_t e = NOTE(cudaMallocAsync(&tmp, prio_bytes + 256 + (size_t)n_seq * 4, stream));
   if (e != cudaSuccess) {
     cudaGetLastError();
     return from_cuda(e);
   }
   float* prio = static_cast<float*>(tmp);
   int32_t* plen_dev = reinterpret_cast<int32_t*>(static_cast<char*>(tmp) + ((prio_bytes + 255) & ~size_t(255)));
-  e = cudaMemcpyAsync(plen_dev, plen_host, (size_t)n_seq * 4, cudaMemcpyHostToDevice, stream);
+  e = NOTE(cudaMemcpyAsync(plen_dev, plen_host, (size_t)n_seq * 4, cudaMemcpyHostToDevice, stream));
   if (e == cudaSuccess)
-    e = launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream);
+    e = NOTE(launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream));
   // the host copy of the lengths must outlive the async copy
-  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   cudaError_t e2 = cudaFreeAsync(tmp, stream);
   if (e == cudaSuccess) e = e2;
   return poison_on(c, e);
@@ -286,10 +330,10 @@ kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, c
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
   if (!q || !k || !v) return KVPOP_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(override_) ||
-      !aligned16(evict_info) || !aligned16(score_out))
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned4(override_) ||
+      !aligned4(evict_info) || !aligned4(score_out))
     return KVPOP_ERR_ALIGN;
-  return poison_on(c, launch_ingest(c->st, c->dm, q, k, v, override_, evict_info, score_out, stream));
+  return poison_on(c, NOTE(launch_ingest(c->st, c->dm, q, k, v, override_, evict_info, score_out, stream)));
 }
 
 kvpop_status kvpop_decode_attend(kvpop_cache* c, const void* q, float* out, cudaStream_t stream) {
@@ -297,7 +341,9 @@ kvpop_status kvpop_decode_attend(kvpop_cache* c, const void* q, float* out, cuda
   if (s != KVPOP_OK) return s;
   if (!q || !out) return KVPOP_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out)) return KVPOP_ERR_ALIGN;
-  return poison_on(c, launch_attend(c->st, c->dm, q, out, c->attend_grid, stream));
+  if (c->use_tc)
+    return poison_on(c, NOTE(tc_launch(c->st, c->dm, tc_map_ptr(c), q, out, c->attend_grid, stream)));
+  return poison_on(c, NOTE(launch_attend(c->st, c->dm, q, out, c->attend_grid, stream)));
 }
 
 kvpop_status kvpop_decode_step(kvpop_cache* c, const void* q, const void* k, const void* v,
@@ -318,24 +364,24 @@ kvpop_status kvpop_decode_step_host(kvpop_cache* c, const void* q, const void* k
   if (s != KVPOP_OK) return s;
   if (!q || !k || !v || !out) return KVPOP_ERR_INVALID_ARG;
   const size_t pairs = c->dm.pairs, d = c->dm.d, G = c->dm.G;
-  cudaError_t e = cudaMemcpyAsync(c->stage_q, q, pairs * G * d * c->esz, cudaMemcpyHostToDevice, stream);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(c->stage_k, k, pairs * d * c->esz, cudaMemcpyHostToDevice, stream);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(c->stage_v, v, pairs * d * c->esz, cudaMemcpyHostToDevice, stream);
+  cudaError_t e = NOTE(cudaMemcpyAsync(c->stage_q, q, pairs * G * d * c->esz, cudaMemcpyHostToDevice, stream));
+  if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_k, k, pairs * d * c->esz, cudaMemcpyHostToDevice, stream));
+  if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_v, v, pairs * d * c->esz, cudaMemcpyHostToDevice, stream));
   if (e != cudaSuccess) return poison_on(c, e);
   s = kvpop_decode_step(c, c->stage_q, c->stage_k, c->stage_v, c->stage_out, nullptr, nullptr,
                         nullptr, stream);
   if (s != KVPOP_OK) return s;
-  e = cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream);
+  e = NOTE(cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream));
   return poison_on(c, e);
 }
 
 kvpop_status kvpop_check(kvpop_cache* c, cudaStream_t stream) {
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
-  cudaError_t e = cudaStreamSynchronize(stream);
+  cudaError_t e = NOTE(cudaStreamSynchronize(stream));
   if (e != cudaSuccess) return poison_on(c, e);
   int32_t err[16];
-  e = cudaMemcpy(err, c->st.err, sizeof(err), cudaMemcpyDeviceToHost);
+  e = NOTE(cudaMemcpy(err, c->st.err, sizeof(err), cudaMemcpyDeviceToHost));
   if (e != cudaSuccess) return poison_on(c, e);
   if (err[0] != 0) {
     cudaMemset(c->st.err, 0, sizeof(err));
@@ -360,10 +406,10 @@ kvpop_status kvpop_export_state(kvpop_cache* c, void* host_buf, size_t* bytes, c
   size_t off = sizeof(hdr) + sizeof(kvpop_config);
   cudaError_t e = cudaSuccess;
   for (auto& b : bufs) {
-    if (e == cudaSuccess) e = cudaMemcpyAsync(out + off, b.ptr, b.bytes, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(out + off, b.ptr, b.bytes, cudaMemcpyDeviceToHost, stream));
     off += b.bytes;
   }
-  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   *bytes = need;
   return poison_on(c, e);
 }
@@ -387,11 +433,11 @@ kvpop_status kvpop_import_state(kvpop_cache* c, const void* host_buf, size_t byt
   size_t off = sizeof(hdr) + sizeof(kvpop_config);
   cudaError_t e = cudaSuccess;
   for (auto& b : bufs) {
-    if (e == cudaSuccess) e = cudaMemcpyAsync(b.ptr, in + off, b.bytes, cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(b.ptr, in + off, b.bytes, cudaMemcpyHostToDevice, stream));
     off += b.bytes;
   }
-  if (e == cudaSuccess) e = cudaMemsetAsync(c->st.part_count, 0, (size_t)c->dm.pairs * 4, stream);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->st.part_count, 0, (size_t)c->dm.pairs * 4, stream));
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   return poison_on(c, e);
 }
 
@@ -400,8 +446,8 @@ kvpop_status kvpop_get_lengths(kvpop_cache* c, int32_t* len_host, cudaStream_t s
   if (s != KVPOP_OK) return s;
   if (!len_host) return KVPOP_ERR_INVALID_ARG;
   std::vector<int32_t> all((size_t)c->dm.pairs);
-  cudaError_t e = cudaMemcpyAsync(all.data(), c->st.len, all.size() * 4, cudaMemcpyDeviceToHost, stream);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  cudaError_t e = NOTE(cudaMemcpyAsync(all.data(), c->st.len, all.size() * 4, cudaMemcpyDeviceToHost, stream));
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   if (e != cudaSuccess) return poison_on(c, e);
   for (int b = 0; b < c->dm.batch; ++b) len_host[b] = all[(size_t)b * c->dm.H];
   return KVPOP_OK;
@@ -414,12 +460,12 @@ kvpop_status kvpop_get_pair_state(kvpop_cache* c, int32_t seq, int32_t head, int
   if (seq < 0 || seq >= c->dm.batch || head < 0 || head >= c->dm.H) return KVPOP_ERR_INVALID_ARG;
   const size_t pair = (size_t)seq * c->dm.H + head, B = c->dm.B;
   cudaError_t e = cudaSuccess;
-  if (pos_host) e = cudaMemcpyAsync(pos_host, c->st.pos + pair * B, B * 4, cudaMemcpyDeviceToHost, stream);
+  if (pos_host) e = NOTE(cudaMemcpyAsync(pos_host, c->st.pos + pair * B, B * 4, cudaMemcpyDeviceToHost, stream));
   if (e == cudaSuccess && score_host)
-    e = cudaMemcpyAsync(score_host, c->st.score + pair * B, B * 4, cudaMemcpyDeviceToHost, stream);
+    e = NOTE(cudaMemcpyAsync(score_host, c->st.score + pair * B, B * 4, cudaMemcpyDeviceToHost, stream));
   if (e == cudaSuccess && nvalid_host)
-    e = cudaMemcpyAsync(nvalid_host, c->st.nvalid + pair, 4, cudaMemcpyDeviceToHost, stream);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    e = NOTE(cudaMemcpyAsync(nvalid_host, c->st.nvalid + pair, 4, cudaMemcpyDeviceToHost, stream));
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   return poison_on(c, e);
 }
 

@@ -1,21 +1,26 @@
 // Decode steps 1-4: ingest the new token, run the delayed scorer on the token
 // that leaves the window, keep or drop it under the fixed budget, scatter it.
 //
-// One CTA owns one KV head h and SB consecutive sequences, so the head's scorer
-// weights W1 [3d][F] are read once per SB sequences.  Warp i of the CTA handles
-// sequence i of the group for the per-sequence work (window ring, eviction).
+// One CTA owns one KV head h and SB consecutive sequences, so each row of the
+// head's scorer weights W1 [3d][F] that it streams feeds SB sequences.  W1 is
+// staged through shared memory in 32 KB chunks by 1-D TMA bulk copies, the
+// first ones issued before the window bookkeeping so the copy overlaps it.
+// Warp i of the CTA does the per-sequence work of sequence i of the group.
 //
 // Paper correspondence: eligible set and the newly eligible token u = p - w
 // (Sec. 3.1, Eq. 4); delayed scoring (Sec. 3.3, App. E.4) with the stateless
 // MLP of Sec. 3.3 / App. E.2 on [k_u; v_u; qbar_u]; static priority
 // (App. B.3); running top-k under the budget (Sec. 3.2, App. C.1).
-#include "kvpop_internal.cuh"
+#include "kvpop_argmin.cuh"
 
 namespace kvpop {
 namespace {
 
-constexpr int SB = 8;          // sequences per CTA (one warp each)
-constexpr int NT = 256;        // threads per CTA
+constexpr int SB = 8;               // sequences per CTA (one warp each)
+constexpr int NT = 256;             // threads per CTA
+constexpr int STG = 3;              // W1 chunk stages
+constexpr int CHUNK = 32768;        // bytes per W1 chunk
+constexpr int MAXF = 1024 / NT;     // hidden units per thread (F <= 1024)
 
 template <typename T>
 struct IngestArgs {
@@ -29,47 +34,47 @@ struct IngestArgs {
   float* score_out;            // [b][H] or nullptr
 };
 
-// Lowest-priority slot over [s, B), ties -> lowest index.  The value of slot
-// `j_new` is taken as `v_new` (it was just written by this warp).
-__device__ __forceinline__ void warp_argmin(const float* __restrict__ sc, int s, int B,
-                                            int j_new, float v_new, float& mval, int& midx) {
-  const int lane = threadIdx.x & 31;
-  float best = INFINITY;
-  int bi = 0x7fffffff;
-  for (int i = s + lane; i < B; i += 32) {
-    float x = (i == j_new) ? v_new : sc[i];
-    if (bi == 0x7fffffff || x < best) { best = x; bi = i; }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    float ob = __shfl_xor_sync(0xffffffffu, best, off);
-    int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-    if (oi != 0x7fffffff && (bi == 0x7fffffff || ob < best || (ob == best && oi < bi))) {
-      best = ob;
-      bi = oi;
-    }
-  }
-  mval = best;
-  midx = bi;
+__host__ __device__ inline size_t ingest_smem_bytes(int d, int Fp, int esz) {
+  return (size_t)STG * CHUNK + ((size_t)3 * d * SB + (size_t)SB * d + (size_t)SB * Fp) * 4 +
+         2 * (size_t)SB * d * esz;
 }
 
 template <typename T>
 __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
   const Dims& dm = a.dm;
-  const int d = dm.d, D = dm.D, G = dm.G, F = dm.F, B = dm.B, H = dm.H;
+  const int d = dm.d, D = dm.D, G = dm.G, F = dm.F, Fp = dm.Fp, B = dm.B, H = dm.H;
   const int h = blockIdx.y;
   const int b0 = blockIdx.x * SB;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int in_dim = 3 * d;
+  const int KC = CHUNK / (Fp * 4);                 // W1 rows per chunk
+  const int nchunks = (in_dim + KC - 1) / KC;
 
-  extern __shared__ __align__(16) unsigned char smem[];
-  float* Xt = reinterpret_cast<float*>(smem);                // [3d][SB] scorer inputs
-  float* qm = Xt + SB * in_dim;                              // [SB][d]
-  float* contrib = qm + SB * d;                              // [SB][F]
-  T* rawk = reinterpret_cast<T*>(contrib + SB * F);          // [SB][d]
-  T* rawv = rawk + SB * d;                                   // [SB][d]
+  extern __shared__ __align__(128) unsigned char smem[];
+  float* Wst = reinterpret_cast<float*>(smem);                         // [STG][KC][Fp]
+  float* Xt = reinterpret_cast<float*>(smem + (size_t)STG * CHUNK);    // [3d][SB]
+  float* qm = Xt + SB * in_dim;                                        // [SB][d]
+  float* contrib = qm + SB * d;                                        // [SB][Fp]
+  T* rawk = reinterpret_cast<T*>(contrib + SB * Fp);                   // [SB][d]
+  T* rawv = rawk + SB * d;
+  __shared__ __align__(8) uint64_t bars[STG];
   __shared__ int s_p[SB];
   __shared__ int s_active[SB];
+
+  const float* W1h = a.st.W1 + (size_t)h * in_dim * Fp;
+  auto issue = [&](int c) {
+    const int rows = min(KC, in_dim - c * KC);
+    const uint32_t bytes = (uint32_t)rows * Fp * 4;
+    const uint32_t bar = smem_u32(&bars[c % STG]);
+    mbar_arrive_expect_tx(bar, bytes);
+    bulk_g2s(smem_u32(Wst + (size_t)(c % STG) * (CHUNK / 4)), W1h + (size_t)c * KC * Fp, bytes, bar);
+  };
+  int issued = 0;
+  if (tid == 0) {
+    for (int s = 0; s < STG; ++s) mbar_init(smem_u32(&bars[s]), 1);
+    mbar_fence_init();
+    for (; issued < min(STG, nchunks); ++issued) issue(issued);
+  }
 
   T* slotK = static_cast<T*>(a.st.slotK);
   T* slotV = static_cast<T*>(a.st.slotV);
@@ -78,7 +83,7 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
 
   // ---- phase 1: per-sequence window bookkeeping and scorer input -------------------
   // X is stored transposed, Xt[i][SB], so phase 2 reads SB inputs with two 16-B loads.
-  if (warp < SB) {
+  {
     const int b = b0 + warp;
     int p = -1, active = 0;
     if (b < dm.batch) {
@@ -101,14 +106,30 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
       const T* rv = ringV + ((size_t)pair * D + ri) * d;
       const float* rq = a.st.ringQm + (size_t)pair * D * d;
       for (int i = lane; i < d; i += 32) {
-        T kk = rk[i], vv = rv[i];
+        const T kk = rk[i], vv = rv[i];
         rawk[warp * d + i] = kk;
         rawv[warp * d + i] = vv;
         Xt[i * SB + warp] = to_f(kk);
         Xt[(d + i) * SB + warp] = to_f(vv);
         // qbar_u: queries u+1 .. p in position order, averaged over D (and G above)
         float acc = 0.f;
-        for (int j = 1; j < D; ++j) acc += rq[((ri + j) % D) * d + i];
+        int j = 1;
+        for (; j + 7 < D; j += 8) {
+          float vals[8];
+#pragma unroll
+          for (int t = 0; t < 8; ++t) {
+            int jj = ri + j + t;
+            jj = jj >= D ? jj - D : jj;
+            vals[t] = rq[(size_t)jj * d + i];
+          }
+#pragma unroll
+          for (int t = 0; t < 8; ++t) acc += vals[t];
+        }
+        for (; j < D; ++j) {
+          int jj = ri + j;
+          jj = jj >= D ? jj - D : jj;
+          acc += rq[(size_t)jj * d + i];
+        }
         acc += qm[warp * d + i];
         Xt[(2 * d + i) * SB + warp] = acc / (float)D;
       }
@@ -120,12 +141,11 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
   __syncthreads();
 
   // ---- phase 1b: push the new token into the window (after u was read) -------------
-  if (warp < SB) {
+  {
     const int b = b0 + warp;
     if (b < dm.batch) {
       const int pair = b * H + h;
-      const int p = s_p[warp];
-      const int wi = p % D;
+      const int wi = s_p[warp] % D;
       T* dk = ringK + ((size_t)pair * D + wi) * d;
       T* dv = ringV + ((size_t)pair * D + wi) * d;
       float* dq = a.st.ringQm + ((size_t)pair * D + wi) * d;
@@ -139,37 +159,64 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
     }
   }
 
-  // ---- phase 2: scorer MLP hidden layer for the SB sequences -----------------------
-  bool any_active = false;
-  for (int i = 0; i < SB; ++i) any_active |= (s_active[i] != 0);
-  if (any_active) {
-    const float* W1 = a.st.W1 + (size_t)h * in_dim * F;
-    const float* b1 = a.st.b1 + (size_t)h * F;
-    const float* w2 = a.st.w2 + (size_t)h * F;
-    for (int f = threadIdx.x; f < F; f += NT) {
-      float acc[SB];
-      const float bias = b1[f];
+  // ---- phase 2: scorer MLP for the SB sequences, W1 streamed chunk by chunk --------
+  const float* b1 = a.st.b1 + (size_t)h * Fp;
+  const float* w2 = a.st.w2 + (size_t)h * Fp;
+  float acc[MAXF][SB];
 #pragma unroll
-      for (int r = 0; r < SB; ++r) acc[r] = bias;
-#pragma unroll 4
-      for (int i = 0; i < in_dim; ++i) {
-        const float w = __ldg(W1 + (size_t)i * F + f);
+  for (int u = 0; u < MAXF; ++u) {
+    const int f = tid + u * NT;
+    const float bias = f < F ? b1[f] : 0.f;
+#pragma unroll
+    for (int r = 0; r < SB; ++r) acc[u][r] = bias;
+  }
+  bool ok = true;
+  for (int c = 0; c < nchunks; ++c) {
+    const int st = c % STG;
+    if (ok) ok = mbar_wait(smem_u32(&bars[st]), (uint32_t)((c / STG) & 1), a.st.err, DEVERR_TIMEOUT_FULL);
+    if (ok) {
+      const int rows = min(KC, in_dim - c * KC);
+      const float* Wc = Wst + (size_t)st * (CHUNK / 4);
+      for (int r = 0; r < rows; ++r) {
+        const int i = c * KC + r;
         const float4 x0 = *reinterpret_cast<const float4*>(Xt + i * SB);
         const float4 x1 = *reinterpret_cast<const float4*>(Xt + i * SB + 4);
-        acc[0] = fmaf(x0.x, w, acc[0]); acc[1] = fmaf(x0.y, w, acc[1]);
-        acc[2] = fmaf(x0.z, w, acc[2]); acc[3] = fmaf(x0.w, w, acc[3]);
-        acc[4] = fmaf(x1.x, w, acc[4]); acc[5] = fmaf(x1.y, w, acc[5]);
-        acc[6] = fmaf(x1.z, w, acc[6]); acc[7] = fmaf(x1.w, w, acc[7]);
-      }
-      const float wf = w2[f];
 #pragma unroll
-      for (int r = 0; r < SB; ++r) contrib[r * F + f] = wf * gelu_erf(acc[r]);
+        for (int u = 0; u < MAXF; ++u) {
+          const int f = tid + u * NT;
+          if (f < Fp) {
+            const float w = Wc[r * Fp + f];
+            acc[u][0] = fmaf(x0.x, w, acc[u][0]); acc[u][1] = fmaf(x0.y, w, acc[u][1]);
+            acc[u][2] = fmaf(x0.z, w, acc[u][2]); acc[u][3] = fmaf(x0.w, w, acc[u][3]);
+            acc[u][4] = fmaf(x1.x, w, acc[u][4]); acc[u][5] = fmaf(x1.y, w, acc[u][5]);
+            acc[u][6] = fmaf(x1.z, w, acc[u][6]); acc[u][7] = fmaf(x1.w, w, acc[u][7]);
+          }
+        }
+      }
+    }
+    __syncthreads();                  // every thread is done with stage st
+    if (tid == 0 && ok && issued < nchunks) { issue(issued); ++issued; }
+  }
+#pragma unroll
+  for (int u = 0; u < MAXF; ++u) {
+    const int f = tid + u * NT;
+    if (f < Fp) {
+      const float wf = f < F ? w2[f] : 0.f;
+#pragma unroll
+      for (int r = 0; r < SB; ++r) contrib[r * Fp + f] = wf * gelu_erf(acc[u][r]);
+    }
+  }
+  if (tid == 0 && !ok) {
+    // a wait expired: let the copies still in flight land before the CTA exits
+    for (int s = 0; s < STG; ++s) {
+      int last = -1;
+      for (int c = s; c < issued; c += STG) last = c;
+      if (last >= 0) mbar_wait(smem_u32(&bars[s]), (uint32_t)((last / STG) & 1), a.st.err, DEVERR_TIMEOUT_DRAIN);
     }
   }
   __syncthreads();
 
   // ---- phase 3: score, keep-or-drop, scatter ------------------------------------------
-  if (warp >= SB) return;
   const int b = b0 + warp;
   if (b >= dm.batch) return;
   const int pair = b * H + h;
@@ -183,7 +230,7 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
     return;
   }
   float r = 0.f;
-  for (int f = lane; f < F; f += 32) r += contrib[warp * F + f];
+  for (int f = lane; f < F; f += 32) r += contrib[warp * Fp + f];
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) r += __shfl_xor_sync(0xffffffffu, r, off);
   r += a.st.b2[h];
@@ -194,6 +241,9 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
 
   float* sc = a.st.score + (size_t)pair * B;
   int32_t* ps = a.st.pos + (size_t)pair * B;
+  const int NB = min_blocks(B);
+  float* bsc = a.st.blk_score + (size_t)pair * NB;
+  int32_t* bsl = a.st.blk_slot + (size_t)pair * NB;
   const int nv = a.st.nvalid[pair];
   int slot = -1, evicted = -1;
   if (nv < B) {
@@ -210,17 +260,14 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
       dk[i] = rawk[warp * d + i];
       dv[i] = rawv[warp * d + i];
     }
-    const int nv_new = nv < B ? nv + 1 : nv;
-    if (nv_new == B) {                       // full: refresh the cached argmin
-      float mval;
-      int midx;
-      warp_argmin(sc, dm.s, B, slot, prio, mval, midx);
-      if (lane == 0) { a.st.min_score[pair] = mval; a.st.min_slot[pair] = midx; }
-    }
+    if (nv == B)
+      update_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
+    else if (nv + 1 == B)
+      rebuild_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
     if (lane == 0) {
       sc[slot] = prio;
       ps[slot] = u;
-      a.st.nvalid[pair] = nv_new;
+      a.st.nvalid[pair] = nv < B ? nv + 1 : nv;
     }
   }
   if (lane == 0) {
@@ -233,8 +280,7 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
 }  // namespace
 
 static size_t ingest_smem(const Dims& dm) {
-  const size_t esz = dm.dtype == KVPOP_F32 ? 4 : 2;
-  return (size_t)SB * (3 * dm.d + dm.d + dm.F) * 4 + 2 * (size_t)SB * dm.d * esz;
+  return ingest_smem_bytes(dm.d, dm.Fp, dm.dtype == KVPOP_F32 ? 4 : 2);
 }
 
 cudaError_t prepare_ingest(const Dims& dm) {

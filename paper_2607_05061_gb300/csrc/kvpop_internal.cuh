@@ -36,10 +36,12 @@ struct State {                 // device pointers of one cache
   int32_t* len;                // [pairs]         tokens seen (same for all heads of a sequence)
   float* min_score;            // [pairs]         argmin over slots [s, B) when full
   int32_t* min_slot;           // [pairs]
-  // scorer
-  const float* W1;             // [H][3d][F]
-  const float* b1;             // [H][F]
-  const float* w2;             // [H][F]
+  float* blk_score;            // [pairs][NB]     per-block minima (blocks of 64 slots)
+  int32_t* blk_slot;           // [pairs][NB]
+  // scorer (hidden width padded to Fp = F rounded up to 4, zero weights)
+  const float* W1;             // [H][3d][Fp]
+  const float* b1;             // [H][Fp]
+  const float* w2;             // [H][Fp]
   const float* b2;             // [H]
   const float* log_gamma;      // [H] or nullptr
   // attention workspace
@@ -49,7 +51,7 @@ struct State {                 // device pointers of one cache
 };
 
 struct Dims {
-  int batch, H, G, d, B, D, s, F;
+  int batch, H, G, d, B, D, s, F, Fp;
   int dtype;                   // kvpop_dtype
   int pairs;
 };
@@ -70,6 +72,13 @@ cudaError_t attend_config(const Dims& dm, AttendConfig* out);
 cudaError_t launch_attend(const State& st, const Dims& dm, const void* q, float* out,
                           int grid, cudaStream_t stream);
 
+// Tensor-core attention for bf16 K/V (TMA tensor maps over the K/V stores).
+size_t tc_maps_size();
+cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out);
+cudaError_t tc_config(const Dims& dm, AttendConfig* out);
+cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const void* q, float* out,
+                      int grid, cudaStream_t stream);
+
 cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const void* K,
                            const void* V, const int32_t* plen_dev, int first_seq, int n_seq,
                            int Pmax, const float* override_, float* tmp_prio,
@@ -82,7 +91,7 @@ __device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
 // Canonical score: NaN -> -inf, -0 -> +0 (every ranking decision uses it).
 __device__ __forceinline__ float canon_score(float r) {
   if (r != r) return -INFINITY;
-  return r + 0.0f;   // -0 + +0 = +0 under round-to-nearest
+  return __fadd_rn(r, 0.0f);   // -0 + +0 = +0 under round-to-nearest
 }
 
 // Static priority (App. B.3, decay step n = 1) in explicit fp32 ops.

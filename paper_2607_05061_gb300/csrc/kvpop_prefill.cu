@@ -13,7 +13,7 @@
 // on the order-preserving bit pattern of the fp32 priority, ties resolved by
 // position -- writes them to slots 0.. in ascending position, and loads the
 // window with the last min(P, D) tokens.
-#include "kvpop_internal.cuh"
+#include "kvpop_argmin.cuh"
 
 namespace kvpop {
 namespace {
@@ -118,9 +118,10 @@ __global__ void __launch_bounds__(NT1) prefill_score_kernel(ScoreArgs<T> a) {
   __syncthreads();
 
   // hidden layer and output projection: thread f (and f + NT1, ...) for all UT rows
-  const float* W1 = a.st.W1 + (size_t)h * in_dim * F;
-  const float* b1 = a.st.b1 + (size_t)h * F;
-  const float* w2 = a.st.w2 + (size_t)h * F;
+  const int Fp = dm.Fp;
+  const float* W1 = a.st.W1 + (size_t)h * in_dim * Fp;
+  const float* b1 = a.st.b1 + (size_t)h * Fp;
+  const float* w2 = a.st.w2 + (size_t)h * Fp;
   float part[UT];
 #pragma unroll
   for (int r = 0; r < UT; ++r) part[r] = 0.f;
@@ -131,7 +132,7 @@ __global__ void __launch_bounds__(NT1) prefill_score_kernel(ScoreArgs<T> a) {
     for (int r = 0; r < UT; ++r) acc[r] = bias;
 #pragma unroll 2
     for (int i = 0; i < in_dim; ++i) {
-      const float w = __ldg(W1 + (size_t)i * F + f);
+      const float w = __ldg(W1 + (size_t)i * Fp + f);
       const float4* xr = reinterpret_cast<const float4*>(Xt + i * UT);
 #pragma unroll
       for (int r4 = 0; r4 < UT / 4; ++r4) {
@@ -303,32 +304,31 @@ __global__ void __launch_bounds__(NT2) prefill_select_kernel(SelectArgs<T> a) {
     }
   }
   __syncthreads();
-  if (warp == 0) {
-    if (nkept == B) {
-      // lowest-priority long-range slot, ties -> lowest index
-      float best = INFINITY;
-      int bi = 0x7fffffff;
-      for (int i = s + lane; i < B; i += 32) {
-        const float x = sc[i];
-        if (bi == 0x7fffffff || x < best) { best = x; bi = i; }
-      }
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ob = __shfl_xor_sync(0xffffffffu, best, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        if (oi != 0x7fffffff && (bi == 0x7fffffff || ob < best || (ob == best && oi < bi))) {
-          best = ob;
-          bi = oi;
-        }
-      }
-      if (lane == 0) { a.st.min_score[pair] = best; a.st.min_slot[pair] = bi; }
-    } else if (lane == 0) {
-      a.st.min_score[pair] = INFINITY;
-      a.st.min_slot[pair] = -1;
+  if (nkept == B) {
+    // block minima over the long-range slots, then the head minimum
+    const int NB = min_blocks(B);
+    float* bsc = a.st.blk_score + (size_t)pair * NB;
+    int32_t* bsl = a.st.blk_slot + (size_t)pair * NB;
+    for (int k = warp; k < NB; k += NT2 / 32) {
+      float m;
+      int mi;
+      block_min(sc, s, B, k, -1, 0.f, m, mi);
+      if (lane == 0) { bsc[k] = m; bsl[k] = mi; }
     }
-    if (lane == 0) {
-      a.st.nvalid[pair] = nkept;
-      a.st.len[pair] = P;
+    __syncthreads();
+    if (warp == 0) {
+      float m;
+      int mi;
+      blocks_min(bsc, bsl, NB, -1, 0.f, 0, m, mi);
+      if (lane == 0) { a.st.min_score[pair] = m; a.st.min_slot[pair] = mi; }
     }
+  } else if (threadIdx.x == 0) {
+    a.st.min_score[pair] = INFINITY;
+    a.st.min_slot[pair] = -1;
+  }
+  if (threadIdx.x == 0) {
+    a.st.nvalid[pair] = nkept;
+    a.st.len[pair] = P;
   }
 }
 

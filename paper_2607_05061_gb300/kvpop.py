@@ -56,6 +56,7 @@ _SIGS = {
     "kvpop_get_lengths": (ctypes.c_int, [_P, POINTER(c_int32), _P]),
     "kvpop_get_pair_state": (ctypes.c_int, [_P, c_int32, c_int32, POINTER(c_int32), POINTER(c_float),
                                             POINTER(c_int32), _P]),
+    "kvpop_last_error": (ctypes.c_char_p, []),
     "kvpop_debug_fail_alloc_after": (None, [c_int32]),
 }
 for _name, (_res, _args) in _SIGS.items():
@@ -71,7 +72,8 @@ class KVpopError(RuntimeError):
     def __init__(self, status: int, what: str):
         self.status = status
         msg = kvpop_status_string(status).decode()
-        super().__init__(f"{what}: {STATUS.get(status, status)} ({msg})")
+        last = kvpop_last_error().decode()
+        super().__init__(f"{what}: {STATUS.get(status, status)} ({msg})" + (f" [{last}]" if last else ""))
 
 
 def _ck(status: int, what: str):
@@ -190,7 +192,9 @@ def parse_state(blob: bytes, cfg: kvpop_config) -> dict:
               ("ringQm", np.float32, (pairs, D, d), 4), ("score", np.float32, (pairs, B), 4),
               ("pos", np.int32, (pairs, B), 4), ("nvalid", np.int32, (pairs,), 4),
               ("len", np.int32, (pairs,), 4), ("min_score", np.float32, (pairs,), 4),
-              ("min_slot", np.int32, (pairs,), 4)]
+              ("min_slot", np.int32, (pairs,), 4),
+              ("blk_score", np.float32, (pairs, (B + 63) // 64), 4),
+              ("blk_slot", np.int32, (pairs, (B + 63) // 64), 4)]
     off = 4 * 8 + ctypes.sizeof(kvpop_config)
     out = {}
     for name, dt, shape, sz in layout:

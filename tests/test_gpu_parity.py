@@ -57,11 +57,12 @@ def test_tiny_gpu_scorer_against_oracle(cuda_device):
     pairs = all_pairs(cfg)
     steps = cfg.decode_steps
     ref = oracle_pairs(cfg, w, L, steps, pairs)
+    pre = oracle_pairs(cfg, w, L, 0, pairs)                   # oracle state right after prefill
     cache = make_cache(cfg, w)
     gpu_prefill(cache, cfg, L, cuda_device)
     # prefill: kept set agreement and per-slot priorities of the common slots
     agree = []
-    for (b, h), tr in zip(pairs, ref):
+    for (b, h), tr in zip(pairs, pre):
         pos, sc = cache.pair_state(b, h)
         o = set(tr.cache.kept_positions())
         agree.append(len(o & set(pos)) / max(1, len(o)))
@@ -79,6 +80,7 @@ def test_tiny_gpu_scorer_against_oracle(cuda_device):
         n_all += steps
     print(f"tiny: prefill kept-set agreement {np.mean(agree):.4f}; "
           f"decode eviction agreement with GPU scores {n_same / n_all:.4f}")
+    assert np.mean(agree) >= 0.99
     cache.free()
 
 
@@ -256,8 +258,13 @@ def test_misaligned_and_bad_arguments(cuda_device):
     with pytest.raises(kvpop.KVpopError) as ei:
         c.attend(buf, out.data_ptr() + 4)
     assert ei.value.status == 2
+    Qp = torch.zeros((2, 32, 16, 128), dtype=torch.bfloat16, device=cuda_device)
+    Kp = torch.zeros((2, 8, 16, 128), dtype=torch.bfloat16, device=cuda_device)
     with pytest.raises(kvpop.KVpopError) as ei:
-        c.prefill(buf, buf, buf, [10, 10])          # two sequences in a batch of one
+        c.prefill(Qp, Kp, Kp, [10, 10])             # two sequences in a batch of one
+    assert ei.value.status == 1
+    with pytest.raises(kvpop.KVpopError) as ei:
+        c.prefill(Qp[:1], Kp[:1], Kp[:1], [17])     # prompt longer than Pmax
     assert ei.value.status == 1
     c.check()
     c.free()
