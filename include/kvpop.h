@@ -168,6 +168,33 @@ kvpop_status kvpop_get_pair_state(kvpop_cache* cache, int32_t seq, int32_t head,
                                   int32_t* pos_host, float* score_host, int32_t* nvalid_host,
                                   cudaStream_t stream);
 
+/* Allocation-free decode attention (no counterpart in the paper: it is an
+ * interface convenience).  For callers that may not allocate device memory
+ * when they decode -- a serving loop whose device memory is fixed up front and
+ * must not grow or stall mid-generation, or a plugin that may only use buffers
+ * its host framework hands it.  Computes the same output as
+ * kvpop_decode_attend (the CUDA-core kernel, for either dtype) over K/V state
+ * the caller owns, and takes the kernel's split-K scratch from a fixed 2 MiB
+ * array compiled into the library instead of calling cudaMalloc; nothing it
+ * calls allocates.
+ *   slotK/slotV [b][H][B][d], ringK/ringV [b][H][D][d] (window entry of
+ *   position t at index t % D), nvalid/len [b][H] int32 (used slots, tokens
+ *   seen), q [b][H*G][d], out [b][H*G][d] fp32 -- all device pointers.
+ * Returns KVPOP_ERR_INVALID_ARG (and a kvpop_last_error message) when
+ * b * H > 12288 or the scratch would exceed the array.  The first call on each
+ * device does a one-time set-up (the array's device address, kernel
+ * attributes) with that device current; make that first call before any
+ * stream capture.  Every call on a device shares the one array and the array
+ * keeps the last call's contents, so calls that overlap on the GPU race:
+ * serialise them. */
+kvpop_status kvpop_attend_noalloc(const void* slotK_dev, const void* slotV_dev,
+                                  const void* ringK_dev, const void* ringV_dev,
+                                  const int32_t* nvalid_dev, const int32_t* len_dev,
+                                  const void* q_dev, float* out_dev, int32_t batch,
+                                  int32_t n_kv_heads, int32_t q_per_kv, int32_t head_dim,
+                                  int32_t budget_B, int32_t delay_D, kvpop_dtype kv_dtype,
+                                  cudaStream_t stream);
+
 /* Description of the last failing CUDA call made by this library on the
  * calling thread ("" if none): call site, error name and message. */
 const char* kvpop_last_error(void);

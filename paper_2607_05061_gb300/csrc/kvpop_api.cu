@@ -138,6 +138,11 @@ std::vector<StateBuf> state_buffers(kvpop_cache* c) {
 
 }  // namespace
 
+namespace kvpop {
+// Message for kvpop_last_error() from other translation units of the library.
+void note_error(const char* msg) { std::snprintf(g_last_error, sizeof(g_last_error), "%s", msg); }
+}
+
 extern "C" {
 
 const char* kvpop_status_string(kvpop_status s) {

@@ -56,6 +56,8 @@ _SIGS = {
     "kvpop_get_lengths": (ctypes.c_int, [_P, POINTER(c_int32), _P]),
     "kvpop_get_pair_state": (ctypes.c_int, [_P, c_int32, c_int32, POINTER(c_int32), POINTER(c_float),
                                             POINTER(c_int32), _P]),
+    "kvpop_attend_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, c_int32, c_int32, c_int32,
+                                            c_int32, c_int32, c_int32, ctypes.c_int, _P]),
     "kvpop_last_error": (ctypes.c_char_p, []),
     "kvpop_debug_fail_alloc_after": (None, [c_int32]),
 }
