@@ -28,7 +28,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decode tokens/sec at 1 GB300 (batch x steps) and achieved HBM GB/s"
 DEFAULT_CONFIG = "cr8x"
-ATTEND_SRC = os.path.join(ROOT, "paper_2607_05061_gb300", "csrc", "kvpop_attend.cu")
+CSRC = os.path.join(ROOT, "paper_2607_05061_gb300", "csrc")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attend_kernel_traffic.txt")
 FALLBACK_HBM_GBS = 6800.0
 
@@ -109,8 +109,12 @@ def committed_traffic(config_name: str):
         for line in f:
             parts = line.split()
             if len(parts) >= 2 and not line.startswith("#"):
-                kv[parts[0]] = parts[1]
-    sha = hashlib.sha256(open(ATTEND_SRC, "rb").read()).hexdigest()
+                kv[parts[0]] = parts[1:] if parts[0] == "source_files" else parts[1]
+    h = hashlib.sha256()
+    for rel in kv.get("source_files", []):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    sha = h.hexdigest()
     if kv.get("source_sha256") != sha or kv.get("config") != config_name:
         return None
     try:
@@ -325,7 +329,9 @@ def run_kvpop(args):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "steps_per_s": 1e3 / step_ms,
         "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": "attend_kernel", "achieved": achieved, "peak": peak,
+        "roofline": {"bound": "hbm", "kernel": ("attend_tc_kernel" if cfg.kv_dtype == "bf16"
+                                                 else "attend_kernel"),
+                     "achieved": achieved, "peak": peak,
                      "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
                      "frac_of_8tbs_nominal": achieved / 8000.0, "traffic": committed_traffic(cfg.name),

@@ -26,6 +26,10 @@ struct kvpop_cache {
   std::vector<void*> allocs;
   std::vector<unsigned char> tc_maps;   // TMA descriptors of the K/V stores (bf16 path)
   bool use_tc = false;
+  bool use_cluster = false;             // cluster ingest kernel
+  float* W1s = nullptr;                 // slice-major scorer weights for it
+  float* b1s = nullptr;
+  float* w2s = nullptr;
   // staging for kvpop_decode_step_host
   void* stage_q = nullptr;
   void* stage_k = nullptr;
@@ -235,6 +239,15 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
     s = from_cuda(NOTE(tc_make_maps(c->st, dm, tc_map_ptr(c))));
   }
   if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest(dm)));
+  c->use_cluster = cluster_ingest_ok(dm);
+  const size_t FS = cluster_ingest_fs(dm);
+  if (s == KVPOP_OK && c->use_cluster) {
+    s = dev_alloc(c, &p, (H * 8 * I * FS + 2 * H * 8 * FS) * 4);
+    c->W1s = (float*)p;
+    c->b1s = c->W1s + H * 8 * I * FS;
+    c->w2s = c->b1s + H * 8 * FS;
+    if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest_cluster(dm)));
+  }
   if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_prefill(dm)));
   if (s == KVPOP_OK) {
     float* W1 = w;
@@ -252,6 +265,26 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
     if (e == cudaSuccess)
       e = NOTE(cudaMemcpy2DAsync(w2, Fp * 4, sc->w2, F * 4, F * 4, H, cudaMemcpyDefault, stream));
     if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
+    if (c->use_cluster) {
+      // slice-major copy for the cluster kernel: slice r holds hidden units [r*FS, r*FS + FS)
+      const size_t nW = (H * 8 * I * FS + 2 * H * 8 * FS) * 4;
+      if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(c->W1s, 0, nW, stream));
+      for (size_t h = 0; h < H && e == cudaSuccess; ++h)
+        for (size_t r = 0; r < 8 && e == cudaSuccess; ++r) {
+          const size_t f0 = r * FS;
+          if (f0 >= F) break;
+          const size_t wcols = (F - f0 < FS) ? F - f0 : FS;
+          const size_t sl = h * 8 + r;
+          e = NOTE(cudaMemcpy2DAsync(c->W1s + sl * I * FS, FS * 4, sc->W1 + h * I * F + f0, F * 4,
+                                     wcols * 4, I, cudaMemcpyDefault, stream));
+          if (e == cudaSuccess)
+            e = NOTE(cudaMemcpyAsync(c->b1s + sl * FS, sc->b1 + h * F + f0, wcols * 4,
+                                     cudaMemcpyDefault, stream));
+          if (e == cudaSuccess)
+            e = NOTE(cudaMemcpyAsync(c->w2s + sl * FS, sc->w2 + h * F + f0, wcols * 4,
+                                     cudaMemcpyDefault, stream));
+        }
+    }
     if (e == cudaSuccess && sc->log_gamma) {
       e = NOTE(cudaMemcpyAsync(lg, sc->log_gamma, H * 4, cudaMemcpyDefault, stream));
       c->st.log_gamma = lg;
@@ -338,6 +371,9 @@ kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, c
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned4(override_) ||
       !aligned4(evict_info) || !aligned4(score_out))
     return KVPOP_ERR_ALIGN;
+  if (c->use_cluster)
+    return poison_on(c, NOTE(launch_ingest_cluster(c->st, c->dm, c->W1s, c->b1s, c->w2s, q, k, v,
+                                                   override_, evict_info, score_out, stream)));
   return poison_on(c, NOTE(launch_ingest(c->st, c->dm, q, k, v, override_, evict_info, score_out, stream)));
 }
 

@@ -1,0 +1,380 @@
+// Decode steps 1-4 with one thread-block cluster per (KV head, group of 16
+// sequences): ingest, delayed scorer, keep-or-drop, scatter.
+//
+// The 8 CTAs of a cluster split the scorer's hidden units: CTA r holds the
+// slice [r*FS, (r+1)*FS) of W1 (3d x FS fp32, 48 KB for d = 128, F = 256),
+// loaded in one go by bulk copies together with everything its two "owned"
+// sequences need (window query means, the leaving token's K/V row, the new
+// q/k/v).  Each owner builds its sequences' scorer inputs
+// x = [k_u; v_u; qbar_u] (Sec. 3.3 delayed scoring, App. E.4) and writes them
+// into every CTA of the cluster through distributed shared memory; after a
+// cluster barrier each CTA evaluates its hidden slice for all 16 sequences and
+// sends the partial output sums back to the owners; the owners add the 8
+// partials in a fixed order, then run the keep-or-drop rule of Sec. 3.2 /
+// App. C.1 (static priority, App. B.3) and scatter the token into its slot.
+// The state the eviction reads (used slots, the cached minimum, its block) is
+// loaded at kernel start so its latency hides behind the scorer.
+#include "kvpop_argmin.cuh"
+
+namespace kvpop {
+namespace {
+
+constexpr int CS = 8;          // CTAs per cluster (hidden-unit slices)
+constexpr int SBC = 16;        // sequences per cluster
+constexpr int OWN = SBC / CS;  // sequences owned by each CTA (2)
+constexpr int NT = 256;        // threads per CTA: warp w evaluates sequences 2w, 2w+1
+
+template <typename T>
+struct ClArgs {
+  State st;
+  Dims dm;
+  const float* W1s;            // [H][CS][3d][FS]
+  const float* b1s;            // [H][CS][FS]
+  const float* w2s;            // [H][CS][FS]
+  int FS;
+  const T* q;                  // [b][H*G][d]
+  const T* k;                  // [b][H][d]
+  const T* v;
+  const float* override_;
+  int32_t* evict_info;
+  float* score_out;
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+struct ClLayout {              // byte offsets into dynamic shared memory
+  int ws, x, qm, qrow, kvrow, newkv, part, total;
+};
+__host__ __device__ inline ClLayout cl_layout(int d, int D, int G, int FS, int esz) {
+  ClLayout L;
+  const int R = d * esz;
+  int o = 0;
+  L.ws = o;    o += 3 * d * FS * 4;                 // W1 slice, then b1, w2 slices
+  o += 2 * FS * 4;
+  L.x = o;     o += SBC * 3 * d * 4;                // scorer inputs of the 16 sequences
+  L.qm = o;    o += OWN * D * d * 4;                // window query means of the owned sequences
+  L.qrow = o;  o += OWN * G * R;                    // new queries
+  L.kvrow = o; o += OWN * 2 * R;                    // K, V row of the leaving token
+  L.newkv = o; o += OWN * 2 * R;                    // new K, V row
+  L.part = o;  o += CS * OWN * 4;                   // partial scores from each CTA
+  L.total = o;
+  return L;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
+  const Dims& dm = a.dm;
+  const int d = dm.d, D = dm.D, G = dm.G, F = dm.F, B = dm.B, H = dm.H, FS = a.FS;
+  const int in_dim = 3 * d;
+  const int R = d * (int)sizeof(T);
+  const int h = blockIdx.y;
+  const uint32_t rank = cluster_rank();
+  const int group = blockIdx.x / CS;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const ClLayout L = cl_layout(d, D, G, FS, (int)sizeof(T));
+
+  extern __shared__ __align__(128) unsigned char smem[];
+  float* Ws = reinterpret_cast<float*>(smem + L.ws);
+  const float* b1s = Ws + in_dim * FS;
+  const float* w2s = b1s + FS;
+  float* X = reinterpret_cast<float*>(smem + L.x);           // [SBC][3d]
+  float* rqm = reinterpret_cast<float*>(smem + L.qm);        // [OWN][D][d]
+  T* qrow = reinterpret_cast<T*>(smem + L.qrow);             // [OWN][G][d]
+  T* kvrow = reinterpret_cast<T*>(smem + L.kvrow);           // [OWN][2][d]
+  T* newkv = reinterpret_cast<T*>(smem + L.newkv);           // [OWN][2][d]
+  float* part = reinterpret_cast<float*>(smem + L.part);     // [CS][OWN]
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int s_p[OWN];
+
+  // sequences of this cluster: group*SBC + j; CTA `rank` owns j = OWN*rank + o
+  const int own_b0 = group * SBC + OWN * (int)rank;
+
+  // ---- issue every load this CTA needs ------------------------------------------------
+  if (tid == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    mbar_fence_init();
+    const uint32_t bb = smem_u32(&bar);
+    const size_t slice = (size_t)h * CS + rank;
+    const uint32_t wbytes = (uint32_t)(in_dim * FS * 4), vbytes = (uint32_t)(FS * 4);
+    mbar_expect_tx(bb, wbytes + 2 * vbytes);
+    const unsigned char* wsrc = reinterpret_cast<const unsigned char*>(a.W1s + slice * in_dim * FS);
+    for (uint32_t off = 0; off < wbytes; off += 16384)
+      bulk_g2s(smem_u32(smem + L.ws + off), wsrc + off, min(16384u, wbytes - off), bb);
+    bulk_g2s(smem_u32(Ws + in_dim * FS), a.b1s + slice * FS, vbytes, bb);
+    bulk_g2s(smem_u32(Ws + in_dim * FS + FS), a.w2s + slice * FS, vbytes, bb);
+    uint32_t rest = 0;
+    for (int o = 0; o < OWN; ++o) {
+      const int b = own_b0 + o;
+      s_p[o] = -1;
+      if (b >= dm.batch) continue;
+      const int pair = b * H + h;
+      const int p = a.st.len[pair];
+      s_p[o] = p;
+      rest += (uint32_t)(D * d * 4 + G * R + 4 * R);
+    }
+    mbar_arrive_expect_tx(bb, rest);
+    for (int o = 0; o < OWN; ++o) {
+      const int b = own_b0 + o;
+      if (b >= dm.batch) continue;
+      const int pair = b * H + h;
+      const int ri = s_p[o] % D;
+      bulk_g2s(smem_u32(rqm + (size_t)o * D * d), a.st.ringQm + (size_t)pair * D * d, D * d * 4, bb);
+      bulk_g2s(smem_u32(qrow + (size_t)o * G * d), a.q + (size_t)pair * G * d, G * R, bb);
+      bulk_g2s(smem_u32(kvrow + (size_t)(2 * o) * d),
+               static_cast<const T*>(a.st.ringK) + ((size_t)pair * D + ri) * d, R, bb);
+      bulk_g2s(smem_u32(kvrow + (size_t)(2 * o + 1) * d),
+               static_cast<const T*>(a.st.ringV) + ((size_t)pair * D + ri) * d, R, bb);
+      bulk_g2s(smem_u32(newkv + (size_t)(2 * o) * d), a.k + (size_t)pair * d, R, bb);
+      bulk_g2s(smem_u32(newkv + (size_t)(2 * o + 1) * d), a.v + (size_t)pair * d, R, bb);
+    }
+  }
+  // eviction state of the owned sequences, read now so it is ready later
+  int ev_nv = 0, ev_mslot = -1;
+  float ev_mscore = INFINITY;
+  if (warp < OWN) {
+    const int b = own_b0 + warp;
+    if (b < dm.batch) {
+      const int pair = b * H + h;
+      ev_nv = a.st.nvalid[pair];
+      ev_mscore = a.st.min_score[pair];
+      ev_mslot = a.st.min_slot[pair];
+    }
+  }
+  __syncthreads();
+  const bool ok = mbar_wait(smem_u32(&bar), 0, a.st.err, DEVERR_TIMEOUT_FULL);
+
+  // ---- owners: scorer inputs, broadcast to the cluster; window update ------------------
+  if (warp < OWN) {
+    const int o = warp;
+    const int j = OWN * (int)rank + o;       // row of X
+    const int b = own_b0 + o;
+    const int p = s_p[o];
+    const bool active = ok && b < dm.batch && p >= D;
+    const int ri = p >= 0 ? p % D : 0;
+    const uint32_t xrow = smem_u32(X + (size_t)j * in_dim);
+    for (int i4 = lane; i4 < in_dim / 4; i4 += 32) {
+      float4 val = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (active) {
+        float e[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int i = i4 * 4 + t;
+          if (i < d) {
+            e[t] = to_f(kvrow[(2 * o) * d + i]);
+          } else if (i < 2 * d) {
+            e[t] = to_f(kvrow[(2 * o + 1) * d + i - d]);
+          } else {
+            const int c = i - 2 * d;
+            float qsum = 0.f;
+            for (int g = 0; g < G; ++g) qsum += to_f(qrow[(o * G + g) * d + c]);
+            const float qm_p = qsum * (1.0f / (float)G);
+            // qbar_u: queries u+1 .. p in position order, averaged over D
+            float acc = 0.f;
+            for (int jj = 1; jj < D; ++jj) {
+              int w = ri + jj;
+              w = w >= D ? w - D : w;
+              acc += rqm[((size_t)o * D + w) * d + c];
+            }
+            acc += qm_p;
+            e[t] = acc / (float)D;
+          }
+        }
+        val = make_float4(e[0], e[1], e[2], e[3]);
+      }
+#pragma unroll
+      for (int dst = 0; dst < CS; ++dst) st_cluster_v4(map_rank(xrow + i4 * 16, dst), val);
+    }
+    if (ok && b < dm.batch) {
+      // push the new token into the window slot of u (u's copy is in kvrow)
+      const int pair = b * H + h;
+      T* dk = static_cast<T*>(a.st.ringK) + ((size_t)pair * D + ri) * d;
+      T* dv = static_cast<T*>(a.st.ringV) + ((size_t)pair * D + ri) * d;
+      float* dq = a.st.ringQm + ((size_t)pair * D + ri) * d;
+      for (int i = lane; i < d; i += 32) {
+        dk[i] = newkv[(2 * o) * d + i];
+        dv[i] = newkv[(2 * o + 1) * d + i];
+        float qsum = 0.f;
+        for (int g = 0; g < G; ++g) qsum += to_f(qrow[(o * G + g) * d + i]);
+        dq[i] = qsum * (1.0f / (float)G);
+      }
+    }
+  }
+  cluster_sync();   // every X row is in every CTA
+
+  // ---- this CTA's hidden slice for all 16 sequences --------------------------------------
+  {
+    const int j0 = 2 * warp, j1 = 2 * warp + 1;
+    const float* x0 = X + (size_t)j0 * in_dim;
+    const float* x1 = X + (size_t)j1 * in_dim;
+    float c0 = 0.f, c1 = 0.f;
+    for (int f = lane; f < FS; f += 32) {
+      float a0 = b1s[f], a1 = a0;
+#pragma unroll 4
+      for (int i = 0; i < in_dim; i += 4) {
+        const float4 u0 = *reinterpret_cast<const float4*>(x0 + i);
+        const float4 u1 = *reinterpret_cast<const float4*>(x1 + i);
+        const float w0 = Ws[(i + 0) * FS + f], w1 = Ws[(i + 1) * FS + f];
+        const float w2 = Ws[(i + 2) * FS + f], w3 = Ws[(i + 3) * FS + f];
+        a0 = fmaf(u0.x, w0, a0); a0 = fmaf(u0.y, w1, a0); a0 = fmaf(u0.z, w2, a0); a0 = fmaf(u0.w, w3, a0);
+        a1 = fmaf(u1.x, w0, a1); a1 = fmaf(u1.y, w1, a1); a1 = fmaf(u1.z, w2, a1); a1 = fmaf(u1.w, w3, a1);
+      }
+      const float wf = w2s[f];
+      c0 = fmaf(wf, gelu_erf(a0), c0);
+      c1 = fmaf(wf, gelu_erf(a1), c1);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      c0 += __shfl_xor_sync(0xffffffffu, c0, off);
+      c1 += __shfl_xor_sync(0xffffffffu, c1, off);
+    }
+    // sequences 2w, 2w+1 are owned by CTA w (OWN = 2): part[rank][o] there
+    if (lane == 0) {
+      const uint32_t dst = (uint32_t)warp;
+      st_cluster_f32(map_rank(smem_u32(part + rank * OWN + 0), dst), c0);
+      st_cluster_f32(map_rank(smem_u32(part + rank * OWN + 1), dst), c1);
+    }
+  }
+  cluster_sync();   // partial sums have arrived; no remote access after this point
+  if (tid == 0 && !ok) {
+    // a wait expired: let the copies still in flight land before the CTA exits
+    mbar_wait(smem_u32(&bar), 0, a.st.err, DEVERR_TIMEOUT_DRAIN);
+  }
+
+  // ---- owners: score, keep-or-drop, scatter ------------------------------------------------
+  if (warp >= OWN) return;
+  const int o = warp;
+  const int b = own_b0 + o;
+  if (b >= dm.batch || !ok) return;
+  const int pair = b * H + h;
+  const int p = s_p[o];
+  if (p < D) {
+    if (lane == 0) {
+      a.st.len[pair] = p + 1;
+      if (a.evict_info) { a.evict_info[2 * pair] = -1; a.evict_info[2 * pair + 1] = -1; }
+      if (a.score_out) a.score_out[pair] = __int_as_float(0x7fc00000);
+    }
+    return;
+  }
+  float r = 0.f;
+  for (int src = 0; src < CS; ++src) r += part[src * OWN + o];
+  r += a.st.b2[h];
+  if (a.override_) r = a.override_[pair];
+  r = canon_score(r);
+  const int u = p - D;
+  const float prio = static_priority(r, u, a.st.log_gamma, h);
+
+  float* sc = a.st.score + (size_t)pair * B;
+  int32_t* ps = a.st.pos + (size_t)pair * B;
+  const int NB = min_blocks(B);
+  float* bsc = a.st.blk_score + (size_t)pair * NB;
+  int32_t* bsl = a.st.blk_slot + (size_t)pair * NB;
+  int slot = -1, evicted = -1;
+  if (ev_nv < B) {
+    slot = ev_nv;
+  } else if (prio > ev_mscore) {
+    slot = ev_mslot;
+    evicted = ps[slot];
+  }
+  if (slot >= 0) {
+    T* dk = static_cast<T*>(a.st.slotK) + ((size_t)pair * B + slot) * d;
+    T* dv = static_cast<T*>(a.st.slotV) + ((size_t)pair * B + slot) * d;
+    for (int i = lane; i < d; i += 32) {
+      dk[i] = kvrow[(2 * o) * d + i];
+      dv[i] = kvrow[(2 * o + 1) * d + i];
+    }
+    if (ev_nv == B)
+      update_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
+    else if (ev_nv + 1 == B)
+      rebuild_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
+    if (lane == 0) {
+      sc[slot] = prio;
+      ps[slot] = u;
+      a.st.nvalid[pair] = ev_nv < B ? ev_nv + 1 : ev_nv;
+    }
+  }
+  if (lane == 0) {
+    a.st.len[pair] = p + 1;
+    if (a.evict_info) { a.evict_info[2 * pair] = slot; a.evict_info[2 * pair + 1] = evicted; }
+    if (a.score_out) a.score_out[pair] = r;
+  }
+  (void)F;
+}
+
+}  // namespace
+
+int cluster_ingest_fs(const Dims& dm) { return ((dm.F + 31) / 32 * 32) / CS; }
+
+bool cluster_ingest_ok(const Dims& dm) {
+  const int FS = cluster_ingest_fs(dm);
+  const ClLayout L = cl_layout(dm.d, dm.D, dm.G, FS, dm.dtype == KVPOP_F32 ? 4 : 2);
+  return FS <= 64 && L.total <= 200 * 1024;
+}
+
+size_t cluster_ingest_smem(const Dims& dm) {
+  return cl_layout(dm.d, dm.D, dm.G, cluster_ingest_fs(dm), dm.dtype == KVPOP_F32 ? 4 : 2).total;
+}
+
+cudaError_t prepare_ingest_cluster(const Dims& dm) {
+  const int smem = (int)cluster_ingest_smem(dm);
+  if (dm.dtype == KVPOP_F32)
+    return cudaFuncSetAttribute(ingest_cluster_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  return cudaFuncSetAttribute(ingest_cluster_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+template <typename T>
+static cudaError_t launch_cl(const State& st, const Dims& dm, const float* W1s, const float* b1s,
+                             const float* w2s, const void* q, const void* k, const void* v,
+                             const float* override_, int32_t* evict_info, float* score_out,
+                             cudaStream_t stream) {
+  ClArgs<T> a{st, dm, W1s, b1s, w2s, cluster_ingest_fs(dm), (const T*)q, (const T*)k,
+              (const T*)v, override_, evict_info, score_out};
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(CS * ((dm.batch + SBC - 1) / SBC), dm.H, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = cluster_ingest_smem(dm);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CS;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, ingest_cluster_kernel<T>, a);
+}
+
+cudaError_t launch_ingest_cluster(const State& st, const Dims& dm, const float* W1s,
+                                  const float* b1s, const float* w2s, const void* q,
+                                  const void* k, const void* v, const float* override_,
+                                  int32_t* evict_info, float* score_out, cudaStream_t stream) {
+  if (dm.dtype == KVPOP_F32)
+    return launch_cl<float>(st, dm, W1s, b1s, w2s, q, k, v, override_, evict_info, score_out, stream);
+  return launch_cl<bf16>(st, dm, W1s, b1s, w2s, q, k, v, override_, evict_info, score_out, stream);
+}
+
+}  // namespace kvpop

@@ -61,6 +61,16 @@ cudaError_t launch_ingest(const State& st, const Dims& dm, const void* q, const 
                           const void* v, const float* override_, int32_t* evict_info,
                           float* score_out, cudaStream_t stream);
 
+// Cluster ingest (8 CTAs per KV head and 16 sequences, hidden units split 8 ways).
+// Weights in slice-major layout: W1s [H][8][3d][FS], b1s / w2s [H][8][FS].
+bool cluster_ingest_ok(const Dims& dm);
+int cluster_ingest_fs(const Dims& dm);
+cudaError_t prepare_ingest_cluster(const Dims& dm);
+cudaError_t launch_ingest_cluster(const State& st, const Dims& dm, const float* W1s,
+                                  const float* b1s, const float* w2s, const void* q,
+                                  const void* k, const void* v, const float* override_,
+                                  int32_t* evict_info, float* score_out, cudaStream_t stream);
+
 // Attention kernel resources for a (dtype, d, G) combination.
 struct AttendConfig {
   int threads;
