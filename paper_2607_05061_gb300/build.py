@@ -38,6 +38,8 @@ def _compile(src: str, verbose_ptxas: bool) -> str:
     obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
     cmd = [nvcc_path(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
            "--expt-relaxed-constexpr", "-c", os.path.join(CSRC, src), "-o", obj]
+    # optional -D overrides of the kernels' compile-time tuning constants
+    cmd[1:1] = os.environ.get("KVPOP_NVCC_DEFINES", "").split()
     if verbose_ptxas:
         cmd.insert(1, "-Xptxas=-v")
     r = subprocess.run(cmd, capture_output=True, text=True)

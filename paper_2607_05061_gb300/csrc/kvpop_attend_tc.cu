@@ -6,8 +6,10 @@
 //  * K and V rows arrive by 2-D TMA tensor copies (one box per 64-column half
 //    of a row) with the 128-byte swizzle, so every ldmatrix below reads eight
 //    distinct bank groups.
-//  * Each consumer warp takes 16 keys.  Logits S^T[16 keys x 8] = K Q^T run as
-//    m16n8k16 bf16 MMAs over d (the G <= 4 query heads of the KV head padded to
+//  * Each of the 8 consumer warps takes 16 keys of a 128-key tile (2 stages of
+//    64 KB; a sweep of tile size, stage count and CTAs per SM on GB300 put this
+//    shape at 0.98 of the measured copy bandwidth).  Logits S^T[16 keys x 8] =
+//    K Q^T run as m16n8k16 bf16 MMAs over d (the G <= 4 query heads of the KV head padded to
 //    the N = 8 of the instruction; Q^T fragments stay in registers for the
 //    pair).  The fp32 accumulator is scaled by log2(e)/sqrt(d).
 //  * Online softmax per head with a lazily raised running maximum (only when
@@ -28,14 +30,25 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kThr = 8.0f;
 
+// Pipeline shape (tuned on GB300 for the cr8x decode step).
+#ifndef KVPOP_TC_NWC
+#define KVPOP_TC_NWC 8
+#endif
+#ifndef KVPOP_TC_STAGES
+#define KVPOP_TC_STAGES 2
+#endif
+#ifndef KVPOP_TC_MINBLOCKS
+#define KVPOP_TC_MINBLOCKS 1
+#endif
+
 template <int HD, int G>
 struct TcTraits {
   static constexpr int NH = HD / 64;               // 128-byte column halves per row
   static constexpr int NKS = HD / 16;              // k-steps of the QK contraction
   static constexpr int NMT = HD / 16;              // m-tiles of O^T
-  static constexpr int NWC = 4;                    // consumer warps, 16 keys each
+  static constexpr int NWC = KVPOP_TC_NWC;         // consumer warps, 16 keys each
   static constexpr int TILE = 16 * NWC;
-  static constexpr int STAGES = 6;
+  static constexpr int STAGES = KVPOP_TC_STAGES;
   static constexpr int THREADS = (NWC + 1) * 32;
   static constexpr int HALF_BYTES = TILE * 128;    // one box
   static constexpr int STAGE_BYTES = 2 * NH * HALF_BYTES;
@@ -59,6 +72,7 @@ struct TcArgs {
   int32_t* part_count;
   int32_t* err;
   int pairs, B, D;
+  int ring_rows;               // rows of a window box: min(TILE, D rounded up to 8)
   float qscale;
 };
 
@@ -105,18 +119,17 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 __device__ __forceinline__ void consumer_sync() {
-  asm volatile("bar.sync 1, %0;" ::"r"(4 * 32) : "memory");
+  asm volatile("bar.sync 1, %0;" ::"r"(KVPOP_TC_NWC * 32) : "memory");
 }
 
 template <int HD, int G>
-__global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, 1)
+__global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     attend_tc_kernel(const __grid_constant__ CUtensorMap mapSK, const __grid_constant__ CUtensorMap mapSV,
                      const __grid_constant__ CUtensorMap mapRK, const __grid_constant__ CUtensorMap mapRV,
                      TcArgs a) {
   using Tr = TcTraits<HD, G>;
   constexpr int TILE = Tr::TILE, NH = Tr::NH, NKS = Tr::NKS, NMT = Tr::NMT;
   constexpr int STAGES = Tr::STAGES, NWC = Tr::NWC, NT = Tr::THREADS;
-  static_assert(NWC == 4, "consumer_sync assumes 4 consumer warps");
 
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -170,15 +183,21 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, 1)
         const int nvt = (nv + TILE - 1) / TILE;
         const CUtensorMap *mk, *mv;
         int row;
-        if (lt < nvt) { mk = &mapSK; mv = &mapSV; row = p * a.B + lt * TILE; }
-        else          { mk = &mapRK; mv = &mapRV; row = p * a.D + (lt - nvt) * TILE; }
+        uint32_t bytes;
+        if (lt < nvt) {
+          mk = &mapSK; mv = &mapSV; row = p * a.B + lt * TILE;
+          bytes = (uint32_t)Tr::STAGE_BYTES;
+        } else {
+          mk = &mapRK; mv = &mapRV; row = p * a.D + (lt - nvt) * TILE;
+          bytes = (uint32_t)(2 * NH * a.ring_rows * 128);
+        }
         const int s = (int)(i % STAGES);
         if (i >= STAGES &&
             !mbar_wait(smem_u32(&bars[STAGES + s]), (uint32_t)((i / STAGES - 1) & 1), a.err,
                        DEVERR_TIMEOUT_EMPTY))
           break;
         const uint32_t fb = smem_u32(&bars[s]);
-        mbar_arrive_expect_tx(fb, (uint32_t)Tr::STAGE_BYTES);
+        mbar_arrive_expect_tx(fb, bytes);
         const uint32_t dst = smem_u32(smem + (size_t)s * Tr::STAGE_BYTES);
 #pragma unroll
         for (int hh = 0; hh < NH; ++hh) {
@@ -378,6 +397,13 @@ struct TcMaps {
   CUtensorMap sk, sv, rk, rv;
 };
 
+// Window boxes only need D rows (rounded up to a swizzle atom's 8) when D < TILE.
+static int tc_ring_rows(const Dims& dm) {
+  const int tile = TcTraits<128, 4>::TILE;
+  const int r = (dm.D + 7) / 8 * 8;
+  return r < tile ? r : tile;
+}
+
 cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out) {
   void* fn = nullptr;
   cudaDriverEntryPointQueryResult q;
@@ -388,11 +414,12 @@ cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out) {
   auto enc = reinterpret_cast<EncodeTiledFn>(fn);
   TcMaps* m = static_cast<TcMaps*>(maps_out);
   const int box = TcTraits<128, 4>::TILE;
+  const int rbox = tc_ring_rows(dm);
   const long long srows = (long long)dm.pairs * dm.B, rrows = (long long)dm.pairs * dm.D;
   if ((e = encode_rows(enc, &m->sk, st.slotK, dm.d, srows, box)) != cudaSuccess) return e;
   if ((e = encode_rows(enc, &m->sv, st.slotV, dm.d, srows, box)) != cudaSuccess) return e;
-  if ((e = encode_rows(enc, &m->rk, st.ringK, dm.d, rrows, box)) != cudaSuccess) return e;
-  return encode_rows(enc, &m->rv, st.ringV, dm.d, rrows, box);
+  if ((e = encode_rows(enc, &m->rk, st.ringK, dm.d, rrows, rbox)) != cudaSuccess) return e;
+  return encode_rows(enc, &m->rv, st.ringV, dm.d, rrows, rbox);
 }
 
 size_t tc_maps_size() { return sizeof(TcMaps); }
@@ -427,6 +454,7 @@ cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const v
   a.pairs = dm.pairs;
   a.B = dm.B;
   a.D = dm.D;
+  a.ring_rows = tc_ring_rows(dm);
   a.qscale = kLog2e / sqrtf((float)dm.d);
 #define LAUNCH(HD_, G_)                                                                   \
   if (dm.d == HD_ && dm.G == G_) {                                                        \

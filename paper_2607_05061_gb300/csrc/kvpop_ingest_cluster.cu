@@ -23,6 +23,7 @@ constexpr int CS = 8;          // CTAs per cluster (hidden-unit slices)
 constexpr int SBC = 16;        // sequences per cluster
 constexpr int OWN = SBC / CS;  // sequences owned by each CTA (2)
 constexpr int NT = 256;        // threads per CTA: warp w evaluates sequences 2w, 2w+1
+constexpr int kMaxBlkLanes = 8;  // block minima prefetched per lane (B <= 16384 slots)
 
 template <typename T>
 struct ClArgs {
@@ -68,7 +69,7 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 }
 
 struct ClLayout {              // byte offsets into dynamic shared memory
-  int ws, x, qm, qrow, kvrow, newkv, part, total;
+  int ws, x, qm, qrow, ring, newkv, part, total;
 };
 __host__ __device__ inline ClLayout cl_layout(int d, int D, int G, int FS, int esz) {
   ClLayout L;
@@ -79,7 +80,7 @@ __host__ __device__ inline ClLayout cl_layout(int d, int D, int G, int FS, int e
   L.x = o;     o += SBC * 3 * d * 4;                // scorer inputs of the 16 sequences
   L.qm = o;    o += OWN * D * d * 4;                // window query means of the owned sequences
   L.qrow = o;  o += OWN * G * R;                    // new queries
-  L.kvrow = o; o += OWN * 2 * R;                    // K, V row of the leaving token
+  L.ring = o;  o += OWN * 2 * R;                    // K, V row of the leaving token
   L.newkv = o; o += OWN * 2 * R;                    // new K, V row
   L.part = o;  o += CS * OWN * 4;                   // partial scores from each CTA
   L.total = o;
@@ -105,7 +106,7 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
   float* X = reinterpret_cast<float*>(smem + L.x);           // [SBC][3d]
   float* rqm = reinterpret_cast<float*>(smem + L.qm);        // [OWN][D][d]
   T* qrow = reinterpret_cast<T*>(smem + L.qrow);             // [OWN][G][d]
-  T* kvrow = reinterpret_cast<T*>(smem + L.kvrow);           // [OWN][2][d]
+  T* ring = reinterpret_cast<T*>(smem + L.ring);             // [OWN][2][d]
   T* newkv = reinterpret_cast<T*>(smem + L.newkv);           // [OWN][2][d]
   float* part = reinterpret_cast<float*>(smem + L.part);     // [CS][OWN]
   __shared__ __align__(8) uint64_t bar;
@@ -127,35 +128,54 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
       bulk_g2s(smem_u32(smem + L.ws + off), wsrc + off, min(16384u, wbytes - off), bb);
     bulk_g2s(smem_u32(Ws + in_dim * FS), a.b1s + slice * FS, vbytes, bb);
     bulk_g2s(smem_u32(Ws + in_dim * FS + FS), a.w2s + slice * FS, vbytes, bb);
+    // rows that do not depend on the sequence length first ...
     uint32_t rest = 0;
-    for (int o = 0; o < OWN; ++o) {
-      const int b = own_b0 + o;
-      s_p[o] = -1;
-      if (b >= dm.batch) continue;
-      const int pair = b * H + h;
-      const int p = a.st.len[pair];
-      s_p[o] = p;
-      rest += (uint32_t)(D * d * 4 + G * R + 4 * R);
-    }
-    mbar_arrive_expect_tx(bb, rest);
+    for (int o = 0; o < OWN; ++o)
+      if (own_b0 + o < dm.batch) rest += (uint32_t)(D * d * 4 + G * R + 2 * R);
+    mbar_expect_tx(bb, rest);
     for (int o = 0; o < OWN; ++o) {
       const int b = own_b0 + o;
       if (b >= dm.batch) continue;
       const int pair = b * H + h;
-      const int ri = s_p[o] % D;
       bulk_g2s(smem_u32(rqm + (size_t)o * D * d), a.st.ringQm + (size_t)pair * D * d, D * d * 4, bb);
       bulk_g2s(smem_u32(qrow + (size_t)o * G * d), a.q + (size_t)pair * G * d, G * R, bb);
-      bulk_g2s(smem_u32(kvrow + (size_t)(2 * o) * d),
-               static_cast<const T*>(a.st.ringK) + ((size_t)pair * D + ri) * d, R, bb);
-      bulk_g2s(smem_u32(kvrow + (size_t)(2 * o + 1) * d),
-               static_cast<const T*>(a.st.ringV) + ((size_t)pair * D + ri) * d, R, bb);
       bulk_g2s(smem_u32(newkv + (size_t)(2 * o) * d), a.k + (size_t)pair * d, R, bb);
       bulk_g2s(smem_u32(newkv + (size_t)(2 * o + 1) * d), a.v + (size_t)pair * d, R, bb);
     }
+    // ... then the leaving token's K/V row, whose window index needs the length
+    int pl[OWN];
+    uint32_t rows = 0;
+    for (int o = 0; o < OWN; ++o) {
+      const int b = own_b0 + o;
+      pl[o] = b < dm.batch ? a.st.len[b * H + h] : -1;
+      s_p[o] = pl[o];
+      if (b < dm.batch) rows += (uint32_t)(2 * R);
+    }
+    mbar_arrive_expect_tx(bb, rows);
+    for (int o = 0; o < OWN; ++o) {
+      const int b = own_b0 + o;
+      if (b >= dm.batch) continue;
+      const int pair = b * H + h;
+      const int ri = pl[o] % D;
+      bulk_g2s(smem_u32(ring + (size_t)(2 * o) * d),
+               static_cast<const T*>(a.st.ringK) + ((size_t)pair * D + ri) * d, R, bb);
+      bulk_g2s(smem_u32(ring + (size_t)(2 * o + 1) * d),
+               static_cast<const T*>(a.st.ringV) + ((size_t)pair * D + ri) * d, R, bb);
+    }
   }
-  // eviction state of the owned sequences, read now so it is ready later
-  int ev_nv = 0, ev_mslot = -1;
+  // lengths and eviction state of the owned sequences, read now so they are ready later:
+  // the cached minimum, the 64 priorities of its block, the block minima and the
+  // position it holds (all that a replacement touches)
+  const int NB = min_blocks(B);
+  const int nbl = (NB + 31) / 32;
+  const bool reg_min = nbl <= kMaxBlkLanes;
+  int ev_nv = 0, ev_mslot = -1, ev_pos = -1;
   float ev_mscore = INFINITY;
+  float blkv[2] = {INFINITY, INFINITY};
+  float nbv[kMaxBlkLanes];
+  int nbs[kMaxBlkLanes];
+#pragma unroll
+  for (int t = 0; t < kMaxBlkLanes; ++t) { nbv[t] = INFINITY; nbs[t] = 0x7fffffff; }
   if (warp < OWN) {
     const int b = own_b0 + warp;
     if (b < dm.batch) {
@@ -163,21 +183,39 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
       ev_nv = a.st.nvalid[pair];
       ev_mscore = a.st.min_score[pair];
       ev_mslot = a.st.min_slot[pair];
+      if (ev_nv == B && ev_mslot >= 0 && reg_min) {
+        const float* sc = a.st.score + (size_t)pair * B;
+        const int lo = (ev_mslot / kMinBlock) * kMinBlock;
+        blkv[0] = (lo + lane < B) ? sc[lo + lane] : INFINITY;
+        blkv[1] = (lo + 32 + lane < B) ? sc[lo + 32 + lane] : INFINITY;
+        ev_pos = a.st.pos[(size_t)pair * B + ev_mslot];
+#pragma unroll
+        for (int t = 0; t < kMaxBlkLanes; ++t) {
+          const int k = lane + 32 * t;
+          nbv[t] = (t < nbl && k < NB) ? a.st.blk_score[(size_t)pair * NB + k] : INFINITY;
+          nbs[t] = (t < nbl && k < NB) ? a.st.blk_slot[(size_t)pair * NB + k] : 0x7fffffff;
+        }
+      }
     }
   }
   __syncthreads();
   const bool ok = mbar_wait(smem_u32(&bar), 0, a.st.err, DEVERR_TIMEOUT_FULL);
 
-  // ---- owners: scorer inputs, broadcast to the cluster; window update ------------------
-  if (warp < OWN) {
-    const int o = warp;
+  // ---- scorer inputs of the owned sequences, broadcast to the cluster; window update --
+  // warp w builds a quarter of the input row of owned sequence w / 4
+  {
+    const int o = warp >> 2, qq = warp & 3;
     const int j = OWN * (int)rank + o;       // row of X
     const int b = own_b0 + o;
     const int p = s_p[o];
     const bool active = ok && b < dm.batch && p >= D;
     const int ri = p >= 0 ? p % D : 0;
+    const T* ku = ring + (size_t)(2 * o) * d;                 // the leaving token u = p - D
+    const T* vu = ring + (size_t)(2 * o + 1) * d;
     const uint32_t xrow = smem_u32(X + (size_t)j * in_dim);
-    for (int i4 = lane; i4 < in_dim / 4; i4 += 32) {
+    const int nq4 = in_dim / 16;             // float4s per quarter
+    if (lane < nq4) {
+      const int i4 = qq * nq4 + lane;
       float4 val = make_float4(0.f, 0.f, 0.f, 0.f);
       if (active) {
         float e[4];
@@ -185,9 +223,9 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
         for (int t = 0; t < 4; ++t) {
           const int i = i4 * 4 + t;
           if (i < d) {
-            e[t] = to_f(kvrow[(2 * o) * d + i]);
+            e[t] = to_f(ku[i]);
           } else if (i < 2 * d) {
-            e[t] = to_f(kvrow[(2 * o + 1) * d + i - d]);
+            e[t] = to_f(vu[i - d]);
           } else {
             const int c = i - 2 * d;
             float qsum = 0.f;
@@ -210,12 +248,12 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
       for (int dst = 0; dst < CS; ++dst) st_cluster_v4(map_rank(xrow + i4 * 16, dst), val);
     }
     if (ok && b < dm.batch) {
-      // push the new token into the window slot of u (u's copy is in kvrow)
+      // push the new token into the window slot of u (u's copy stays in smem)
       const int pair = b * H + h;
       T* dk = static_cast<T*>(a.st.ringK) + ((size_t)pair * D + ri) * d;
       T* dv = static_cast<T*>(a.st.ringV) + ((size_t)pair * D + ri) * d;
       float* dq = a.st.ringQm + ((size_t)pair * D + ri) * d;
-      for (int i = lane; i < d; i += 32) {
+      for (int i = qq * 32 + lane; i < d; i += 128) {
         dk[i] = newkv[(2 * o) * d + i];
         dv[i] = newkv[(2 * o + 1) * d + i];
         float qsum = 0.f;
@@ -290,7 +328,6 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
 
   float* sc = a.st.score + (size_t)pair * B;
   int32_t* ps = a.st.pos + (size_t)pair * B;
-  const int NB = min_blocks(B);
   float* bsc = a.st.blk_score + (size_t)pair * NB;
   int32_t* bsl = a.st.blk_slot + (size_t)pair * NB;
   int slot = -1, evicted = -1;
@@ -298,19 +335,52 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
     slot = ev_nv;
   } else if (prio > ev_mscore) {
     slot = ev_mslot;
-    evicted = ps[slot];
+    evicted = reg_min ? ev_pos : ps[slot];
   }
   if (slot >= 0) {
     T* dk = static_cast<T*>(a.st.slotK) + ((size_t)pair * B + slot) * d;
     T* dv = static_cast<T*>(a.st.slotV) + ((size_t)pair * B + slot) * d;
+    const T* ku = ring + (size_t)(2 * o) * d;
+    const T* vu = ring + (size_t)(2 * o + 1) * d;
     for (int i = lane; i < d; i += 32) {
-      dk[i] = kvrow[(2 * o) * d + i];
-      dv[i] = kvrow[(2 * o + 1) * d + i];
+      dk[i] = ku[i];
+      dv[i] = vu[i];
     }
-    if (ev_nv == B)
-      update_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
-    else if (ev_nv + 1 == B)
+    if (ev_nv == B) {
+      if (reg_min) {
+        // block of the replaced slot from the prefetched priorities, then the head minimum
+        const int k = slot / kMinBlock, lo = k * kMinBlock;
+        float bm = INFINITY;
+        int bmi = 0x7fffffff;
+#pragma unroll
+        for (int r2 = 0; r2 < 2; ++r2) {
+          const int i = lo + r2 * 32 + lane;
+          if (i < B && i >= dm.s) lex_min(bm, bmi, i == slot ? prio : blkv[r2], i);
+        }
+        warp_lex_min(bm, bmi);
+        float m = INFINITY;
+        int mi = 0x7fffffff;
+#pragma unroll
+        for (int t = 0; t < kMaxBlkLanes; ++t) {
+          const int kk = lane + 32 * t;
+          if (t < nbl && kk < NB) {
+            if (kk == k) lex_min(m, mi, bm, bmi);
+            else lex_min(m, mi, nbv[t], nbs[t]);
+          }
+        }
+        warp_lex_min(m, mi);
+        if (lane == 0) {
+          bsc[k] = bm;
+          bsl[k] = bmi;
+          a.st.min_score[pair] = m;
+          a.st.min_slot[pair] = mi;
+        }
+      } else {
+        update_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
+      }
+    } else if (ev_nv + 1 == B) {
       rebuild_min(sc, dm.s, B, slot, prio, bsc, bsl, a.st.min_score + pair, a.st.min_slot + pair);
+    }
     if (lane == 0) {
       sc[slot] = prio;
       ps[slot] = u;
