@@ -241,7 +241,7 @@ def run_kvpop(args):
         over["prompt_len"] = args.prompt_len
     cfg = get_config(args.config, **over)
     if cfg.n_layers != 1:
-        raise SystemExit("bench.py times single-layer workloads (tiny, q4b, cr8x, ragged)")
+        return run_stack_bench(args, cfg, rank, local_rank, world, dev, dist)
     L = gen.prompt_lengths(cfg)
     W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
     cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
@@ -352,6 +352,140 @@ def run_kvpop(args):
         dist.destroy_process_group()
 
 
+# ------------------------------------------------------------------ GPU arm, layer stack
+def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
+    """Decode steps of the Qwen3-8B-shaped stack: per layer Q/K/V projections (cuBLAS bf16),
+    one KVpop cache step, output projection and residual; one step = all layers, replayed
+    from a CUDA graph."""
+    import torch
+    from paper_2607_05061_gb300.stack import DecodeStack
+    from workload import gen
+    L = gen.prompt_lengths(cfg)
+    layers = []
+    for l in range(cfg.n_layers):
+        w = gen.stack_weights(cfg, l, device=dev)
+        for k in ("W1", "b1", "w2", "b2"):
+            w[k] = w[k].cpu()
+        layers.append(w)
+    st = DecodeStack(layers, cfg.batch, cfg.hidden, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim,
+                     cfg.budget_B, cfg.delay_D, cfg.scorer_hidden, n_sink=cfg.n_sink, device=dev)
+    group = 4
+    for l in range(cfg.n_layers):
+        for b0 in range(0, cfg.batch, group):
+            nb = min(group, cfg.batch - b0)
+            X = gen.prompt_hidden(cfg, l, b0, nb, 0, max(L[b0:b0 + nb]), device=dev)
+            st.prefill_layer(l, X, L[b0:b0 + nb], first_seq=b0)
+            del X
+    torch.cuda.synchronize()
+    W, K = args.warmup, args.steps
+    n_attn = 32                                   # eager steps timing each attention launch
+    xs = gen.decode_hidden(cfg, L, 0, W + K + n_attn, device=dev)
+    x_in = torch.empty((cfg.batch, cfg.hidden), dtype=torch.bfloat16, device=dev)
+    x_out = torch.empty_like(x_in)
+    st.capture(x_in, x_out)
+    stream = torch.cuda.current_stream()
+    for j in range(W):
+        x_in.copy_(xs[j])
+        st.graph.replay()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(K):
+        x_in.copy_(xs[W + i])
+        st.graph.replay()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    for c in st.caches:
+        c.check()
+    step_ms_local = t_start.elapsed_time(t_end) / K
+    # attention launch durations: eager steps with events around every layer's attention
+    ev = []
+    x = torch.empty_like(x_in)
+    for i in range(n_attn):
+        xcur = xs[W + K + i]
+        for l, (Lw, cache) in enumerate(zip(st.layers, st.caches)):
+            torch.matmul(xcur, Lw["Wq"], out=st.q)
+            torch.matmul(xcur, Lw["Wk"], out=st.k)
+            torch.matmul(xcur, Lw["Wv"], out=st.v)
+            cache.ingest(st.q, st.k, st.v)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            cache.attend(st.q, st.o)
+            e1.record(stream)
+            ev.append((e0, e1))
+            st.o_bf.copy_(st.o)
+            torch.matmul(st.o_bf, Lw["Wo"], out=st.y)
+            torch.add(xcur, st.y, out=x)
+            xcur = x.clone()
+    torch.cuda.synchronize()
+    attn_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    # end to end: host hidden state in (pinned), final hidden state out, per step
+    E = max(1, min(args.e2e_steps, 64))
+    xh = xs[:E].cpu().pin_memory()
+    oh = torch.empty((cfg.batch, cfg.hidden), dtype=torch.bfloat16).pin_memory()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(E):
+        x_in.copy_(xh[i], non_blocking=True)
+        st.graph.replay()
+        oh.copy_(x_out, non_blocking=True)
+        stream.synchronize()
+    e2e_s = (time.perf_counter() - t0) / E
+    step_ms, _ = reduce_max_sum(step_ms_local, 0.0, world, dev)
+    e2e_ms, _ = reduce_max_sum(e2e_s * 1e3, 0.0, world, dev)
+    tokens_per_step = cfg.batch * world
+    bytes_per_launch = statistics.mean(kv_stream_bytes(cfg, L, W + K + i) for i in range(n_attn))
+    proj_bytes = cfg.n_layers * 2 * (cfg.hidden * (cfg.n_q_heads + 2 * cfg.n_kv_heads) * cfg.head_dim
+                                     + cfg.n_q_heads * cfg.head_dim * cfg.hidden)
+    achieved = bytes_per_launch / (attn_ms / 1e3) / 1e9
+    peak, peak_src = measured_peaks()
+    rec = {
+        "metric": METRIC, "value": tokens_per_step / (step_ms / 1e3), "unit": "tokens/s",
+        "n_gpus": world, "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded counter-based generator)",
+        "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
+                   "layers": cfg.n_layers, "hidden": cfg.hidden, "kv_heads": cfg.n_kv_heads,
+                   "q_per_kv": cfg.q_per_kv, "head_dim": cfg.head_dim, "prompt_len": cfg.prompt_len,
+                   "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype,
+                   "projections": "cuBLAS bf16 GEMMs (torch.matmul), fp32 accumulate",
+                   "l2": f"inputs larger than L2: {cfg.n_layers * bytes_per_launch / 1e9:.2f} GB K/V "
+                         f"+ {proj_bytes / 1e9:.2f} GB weights per step",
+                   "graph": "one CUDA graph per step (all layers)",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "steps_per_s": 1e3 / step_ms,
+        "hbm_gbs_step": (cfg.n_layers * bytes_per_launch + proj_bytes) / (step_ms / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "attend_tc_kernel", "achieved": achieved, "peak": peak,
+                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)", "unit": "GB/s",
+                     "frac": achieved / peak, "frac_of_8tbs_nominal": achieved / 8000.0,
+                     "traffic": None, "algorithmic_bytes_per_launch": bytes_per_launch,
+                     "ms_per_launch": attn_ms},
+        "e2e": {"value": tokens_per_step / (e2e_ms / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": cfg.batch * cfg.hidden * 2,
+                "d2h_bytes_per_step": cfg.batch * cfg.hidden * 2, "steps": E,
+                "how": "pinned hidden state in, graph replay, final hidden state out, sync per step"},
+        "gpu_launches": K * cfg.n_layers * 2,
+        "clocks": clk,
+        "cpu_baseline": None,
+        "cpu_baseline_note": ("not run for the stack: the fp64 oracle would have to prefill 36 layers "
+                              "of a 32768-token prompt (about 58 PFLOP of fp64 projections)"),
+    }
+    st.free()
+    if rank == 0:
+        print(json.dumps(rec), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 # ------------------------------------------------------------------ reference arm (oracle)
 def run_reference(args):
     rank, _, world = dist_info()
@@ -360,6 +494,8 @@ def run_reference(args):
     from oracle.run import prefill_pair
     from workload import gen, get_config
     cfg = get_config(args.config)
+    if cfg.n_layers != 1:
+        raise SystemExit("--impl reference times the oracle on single-layer workloads only")
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
     W, K = args.warmup, args.steps

@@ -14,4 +14,7 @@ from .gen import (  # noqa: F401
     prompt_lengths,
     outlier_channels,
     uniform_scores,
+    stack_weights,
+    prompt_hidden,
+    decode_hidden,
 )

@@ -33,7 +33,7 @@ LP = 1 << 20            # positions per (sequence, head) stream
 STREAM_K, STREAM_V, STREAM_Q = 1, 2, 3
 STREAM_W1, STREAM_W2 = 10, 11
 STREAM_LEN, STREAM_OUTLIER = 20, 21
-STREAM_HIDDEN, STREAM_WPROJ = 40, 41
+STREAM_HIDDEN, STREAM_WPROJ, STREAM_DECODE_HIDDEN = 40, 50, 60
 LAYER_STRIDE = 1000     # stream offset between layers of a stack
 
 _CHUNK = 1 << 24        # elements generated per torch pass
@@ -230,3 +230,51 @@ def uniform_scores(seed: int, stream: int, shape, device="cpu", levels: Optional
     else:
         v = (uniform_u32(seed, stream, flat) % levels).to(torch.float32) * 0.25 - 1.0
     return v.view(*shape)
+
+
+# ---------------------------------------------------------------------- projection stack
+def stack_weights(cfg, layer: int, device="cpu") -> dict:
+    """bf16 projections of one layer, N(0, 1/hidden): ``Wq [hidden][Hq*d]``, ``Wk``, ``Wv``
+    ``[hidden][H*d]``, ``Wo [Hq*d][hidden]``; plus that layer's fp32 scorer (CPU)."""
+    hid, d = cfg.hidden, cfg.head_dim
+    shapes = {"Wq": (hid, cfg.n_q_heads * d), "Wk": (hid, cfg.n_kv_heads * d),
+              "Wv": (hid, cfg.n_kv_heads * d), "Wo": (cfg.n_q_heads * d, hid)}
+    out = {}
+    scale = torch.tensor(1.0 / np.sqrt(hid), dtype=torch.float32, device=device)
+    for m, (name, shp) in enumerate(shapes.items()):
+        n = shp[0] * shp[1]
+        t = torch.empty((n,), dtype=torch.bfloat16, device=device)
+        flat = torch.arange(n, dtype=torch.int64, device=device)
+        for c0 in range(0, n, _CHUNK):
+            c1 = min(n, c0 + _CHUNK)
+            t[c0:c1] = (normal_values(cfg.seed, STREAM_WPROJ + m + layer * LAYER_STRIDE,
+                                      flat[c0:c1]) * scale).to(torch.bfloat16)
+        out[name] = t.view(*shp)
+    W1, b1, w2, b2, lg = scorer_weights(cfg, layer)
+    out.update(W1=W1, b1=b1, w2=w2, b2=b2)
+    if cfg.log_gamma != 0.0:
+        out["log_gamma"] = lg
+    return out
+
+
+def prompt_hidden(cfg, layer: int, b0: int, nb: int, t0: int, nt: int, device="cpu") -> torch.Tensor:
+    """Prompt hidden states of one layer ``[nb][nt][hidden]`` bf16, N(0, 1)."""
+    hid = cfg.hidden
+    out = torch.empty((nb, nt, hid), dtype=torch.bfloat16, device=device)
+    ts = torch.arange(t0, t0 + nt, dtype=torch.int64, device=device)
+    for i in range(nb):
+        base = ((b0 + i) * LP + ts) * hid
+        _rows(cfg.seed, STREAM_HIDDEN + layer * LAYER_STRIDE, base, hid, out[i])
+    return out
+
+
+def decode_hidden(cfg, lengths: Sequence[int], step0: int, nsteps: int, device="cpu") -> torch.Tensor:
+    """Input hidden state of every decode step ``[nsteps][b][hidden]`` bf16, N(0, 1)."""
+    hid = cfg.hidden
+    L = torch.tensor(list(lengths), dtype=torch.int64, device=device)
+    steps = torch.arange(step0, step0 + nsteps, dtype=torch.int64, device=device)
+    bs = torch.arange(len(lengths), dtype=torch.int64, device=device)
+    base = ((bs[None, :] * LP + L[None, :] + steps[:, None]) * hid).reshape(-1)
+    out = torch.empty((nsteps, len(lengths), hid), dtype=torch.bfloat16, device=device)
+    _rows(cfg.seed, STREAM_DECODE_HIDDEN, base, hid, out.view(-1, hid))
+    return out
