@@ -1,0 +1,75 @@
+"""Host-side logic of bench.py: multi-rank aggregation (world size 2 over gloo on
+CPU), the algorithmic byte count, sampling of oracle pairs and the committed
+traffic figure."""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import bench
+from workload import get_config
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _rank_main(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    # rank r reports a step time of 1 + r ms and 100 * (r + 1) tokens
+    mx, sm = bench.reduce_max_sum(1.0 + rank, 100.0 * (rank + 1), world, None)
+    q.put((rank, mx, sm))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_reduce_over_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    # max over ranks of the time, sum over ranks of the tokens, the same on every rank
+    assert res == [(0, 2.0, 300.0), (1, 2.0, 300.0)]
+
+
+def test_single_rank_reduce_is_identity():
+    assert bench.reduce_max_sum(3.5, 7.0, 1) == (3.5, 7.0)
+
+
+def test_kv_stream_bytes_counts_slots_and_window():
+    cfg = get_config("cr8x")
+    # steady state: every pair holds B slots + D window keys of 2 * d * 2 bytes
+    full = cfg.batch * cfg.n_kv_heads * (cfg.budget_B + cfg.delay_D) * 2 * cfg.head_dim * 2
+    assert bench.kv_stream_bytes(cfg, [cfg.prompt_len] * cfg.batch, 0) == full
+    # a short sequence keeps all its eligible tokens
+    tiny = get_config("tiny", budget_B=1000)
+    P = 100
+    expect = tiny.n_kv_heads * ((P + 1 - tiny.delay_D) + tiny.delay_D) * 2 * tiny.head_dim * 4
+    assert bench.kv_stream_bytes(tiny, [P], 0) == expect
+
+
+def test_sample_pairs_are_distinct_and_in_range():
+    cfg = get_config("cr8x")
+    pairs = bench.sample_pairs(cfg, 16)
+    assert len(pairs) == len(set(pairs)) == 16
+    assert all(0 <= b < cfg.batch and 0 <= h < cfg.n_kv_heads for b, h in pairs)
+
+
+def test_committed_traffic_requires_matching_config():
+    assert bench.committed_traffic("ragged") is None
+    t = bench.committed_traffic("cr8x")
+    assert t is None or t > 1_000_000_000
