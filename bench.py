@@ -44,6 +44,8 @@ def parse_args(argv=None):
                     help="override the workload's batch (small profiling cases)")
     ap.add_argument("--prompt-len", type=int, default=None,
                     help="override the workload's prompt length (small profiling cases)")
+    ap.add_argument("--scorer", choices=["mlp", "mlstm"], default="mlp",
+                    help="delayed MLP scorer (the workload's) or the stateful mLSTM scorer")
     ap.add_argument("--e2e-steps", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=96)
@@ -175,15 +177,17 @@ class ClockSampler:
 # ------------------------------------------------------------------ oracle (CPU) legs
 def _oracle_pair_job(args):
     """Prefill one (sequence, KV head) in the oracle (untimed), then time n decode steps."""
-    cfg_name, b, h, n_steps = args
+    cfg_name, b, h, n_steps, scorer = args
     import torch
     torch.set_num_threads(1)
-    from oracle.run import prefill_pair
+    from oracle.run import prefill_pair, prefill_pair_mlstm
     from workload import gen, get_config
     cfg = get_config(cfg_name)
-    w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
-    cache = prefill_pair(cfg, w, b, h, L[b])
+    if scorer == "mlstm":
+        cache = prefill_pair_mlstm(cfg, gen.mlstm_weights(cfg), b, h, L[b])
+    else:
+        cache = prefill_pair(cfg, gen.scorer_weights(cfg), b, h, L[b])
     G = cfg.q_per_kv
     q, k, v = gen.decode_inputs(cfg, [L[b]], 0, n_steps, b0=b)
     q = q[:, 0, h * G:(h + 1) * G].double().numpy()
@@ -202,7 +206,7 @@ def sample_pairs(cfg, n):
     return [(i // cfg.n_kv_heads, i % cfg.n_kv_heads) for i in idx]
 
 
-def cpu_baseline(cfg, n_steps: int):
+def cpu_baseline(cfg, n_steps: int, scorer: str = "mlp"):
     """fp64 oracle decode throughput on this host's cores (spawned pool, one pair per core)."""
     import multiprocessing as mp
     cores = max(1, min(os.cpu_count() or 1, 16))
@@ -211,7 +215,7 @@ def cpu_baseline(cfg, n_steps: int):
         os.environ[var] = "1"
     ctx = mp.get_context("spawn")
     with ctx.Pool(len(pairs)) as pool:
-        times = pool.map(_oracle_pair_job, [(cfg.name, b, h, n_steps) for b, h in pairs])
+        times = pool.map(_oracle_pair_job, [(cfg.name, b, h, n_steps, scorer) for b, h in pairs])
     per_pair_step = statistics.mean(times) / n_steps            # seconds per (pair, step)
     step_time = cfg.batch * cfg.n_kv_heads * per_pair_step / len(pairs)
     return {"value": cfg.batch / step_time, "unit": "tokens/s", "cores": len(pairs), "kind": "oracle",
@@ -243,11 +247,20 @@ def run_kvpop(args):
     if cfg.n_layers != 1:
         return run_stack_bench(args, cfg, rank, local_rank, world, dev, dist)
     L = gen.prompt_lengths(cfg)
-    W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
-    cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
-                             cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
-                             n_sink=cfg.n_sink)
+    if args.scorer == "mlstm":
+        cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
+                                 cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, n_sink=cfg.n_sink,
+                                 mlstm=gen.mlstm_weights(cfg))
+        scorer_desc = (f"stateful delayed mLSTM (Hedgehog, C {cfg.head_dim}x{cfg.head_dim // 2} per "
+                       f"head) fp32")
+    else:
+        W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
+        cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
+                                 cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
+                                 n_sink=cfg.n_sink)
+        scorer_desc = f"MLP {cfg.scorer_in}->{cfg.scorer_hidden} GELU->1 fp32"
     # prefill (untimed), a few sequences at a time to bound the prompt buffers
+    t_prefill = 0.0
     group = 8
     for b0 in range(0, cfg.batch, group):
         nb = min(group, cfg.batch - b0)
@@ -256,7 +269,10 @@ def run_kvpop(args):
         Q = gen.q_tokens(cfg, b0, nb, 0, Pm, device=dev)
         K = gen.kv_tokens(cfg, "k", b0, nb, 0, Pm, device=dev)
         V = gen.kv_tokens(cfg, "v", b0, nb, 0, Pm, device=dev)
+        torch.cuda.synchronize()
+        tp = time.perf_counter()
         cache.prefill(Q, K, V, Lg, first_seq=b0)
+        t_prefill += time.perf_counter() - tp
         del Q, K, V
     torch.cuda.synchronize()
 
@@ -324,11 +340,12 @@ def run_kvpop(args):
                    "kv_heads": cfg.n_kv_heads, "q_per_kv": cfg.q_per_kv, "head_dim": cfg.head_dim,
                    "prompt_len": "ragged U[%d,%d]" % cfg.ragged if cfg.ragged else cfg.prompt_len,
                    "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype,
-                   "scorer": f"MLP {cfg.scorer_in}->{cfg.scorer_hidden} GELU->1 fp32",
+                   "scorer": scorer_desc,
                    "l2": f"inputs larger than L2: {bytes_per_launch / 1e9:.3f} GB K/V read per step",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "steps_per_s": 1e3 / step_ms,
         "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
+        "prefill_s": t_prefill,
         "roofline": {"bound": "hbm", "kernel": ("attend_tc_kernel" if cfg.kv_dtype == "bf16"
                                                  else "attend_kernel"),
                      "achieved": achieved, "peak": peak,
@@ -345,7 +362,7 @@ def run_kvpop(args):
     cache.free()
     del q, k, v
     if rank == 0 and not args.no_cpu_baseline:
-        rec["cpu_baseline"] = cpu_baseline(cfg, args.cpu_steps)
+        rec["cpu_baseline"] = cpu_baseline(cfg, args.cpu_steps, args.scorer)
     if rank == 0:
         print(json.dumps(rec), flush=True)
     if world > 1:

@@ -80,6 +80,26 @@ typedef struct {
                               for none; stored priority = r - u * log_gamma   */
 } kvpop_scorer;
 
+/* Stateful delayed mLSTM scorer (App. A, App. E.3, App. E.4), per KV head.
+ * With x = [k; v]: q~ = phi(W_q x), k~ = phi(W_k x), v~ = W_v x, phi the
+ * Hedgehog map [softmax(y); softmax(-y)]; gates i = exp(w_i.x + b_i),
+ * f = sigmoid(w_f.x + b_f); state C <- f C + i k~ v~^T, z <- f z + i k~ (kept
+ * stabilised); after absorbing token p the token u = p - D is scored
+ * r = a . SiLU((q~_u^T C) / (q~_u^T z)) + b.  Host or device fp32 arrays,
+ * copied at init. */
+typedef struct {
+  const float* Wq;         /* [H][2d][d/2]                                    */
+  const float* Wk;         /* [H][2d][d/2]                                    */
+  const float* Wv;         /* [H][2d][d/2]                                    */
+  const float* wi;         /* [H][2d] input-gate weights                      */
+  const float* wf;         /* [H][2d] forget-gate weights                     */
+  const float* bi;         /* [H]                                             */
+  const float* bf;         /* [H]                                             */
+  const float* a;          /* [H][d/2] output projection                      */
+  const float* b;          /* [H]                                             */
+  const float* log_gamma;  /* [H] per-head log decay or NULL (as kvpop_scorer) */
+} kvpop_mlstm_scorer;
+
 typedef struct kvpop_cache kvpop_cache;   /* opaque, library-owned device state */
 
 /* Human-readable name of a status (static string, never NULL). */
@@ -91,6 +111,13 @@ const char* kvpop_status_string(kvpop_status s);
  * Synchronises `stream` before returning.  *out is NULL on failure. */
 kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* scorer,
                               cudaStream_t stream, kvpop_cache** out);
+
+/* As kvpop_init_cache with the mLSTM scorer; cfg->scorer_hidden is ignored.
+ * The cache additionally holds the recurrent state (C, z, m) of every
+ * (sequence, KV head), which prefill builds over the prompt and every decode
+ * step advances by one token (a sequential scan per pair in prefill). */
+kvpop_status kvpop_init_cache_mlstm(const kvpop_config* cfg, const kvpop_mlstm_scorer* scorer,
+                                    cudaStream_t stream, kvpop_cache** out);
 
 /* Release the cache and all its device memory.  kvpop_free(NULL) is KVPOP_OK.
  * Synchronises the device work of the cache first. */

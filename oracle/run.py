@@ -45,13 +45,34 @@ def prefill_pair(cfg, weights, b: int, h: int, prompt_len: int,
     return prefill_head(head_params(cfg, weights, h), Q, K, V, cfg.head_dim, G, prefill_override)
 
 
+def prefill_pair_mlstm(cfg, mw, b: int, h: int, prompt_len: int,
+                       prefill_override: Optional[np.ndarray] = None):
+    from .mlstm import MlstmParams, prefill_mlstm
+    G = cfg.q_per_kv
+    K = _f64(gen.kv_tokens(cfg, "k", b, 1, 0, prompt_len, heads=[h]))[0, 0]
+    V = _f64(gen.kv_tokens(cfg, "v", b, 1, 0, prompt_len, heads=[h]))[0, 0]
+    Q = _f64(gen.q_tokens(cfg, b, 1, 0, prompt_len, heads=range(h * G, (h + 1) * G)))[0]
+    lg = float(np.float32(mw["log_gamma"][h])) if "log_gamma" in mw else 0.0
+    op = OracleParams(np.zeros((3 * cfg.head_dim, 1)), np.zeros(1), np.zeros(1), 0.0,
+                      cfg.budget_B, cfg.delay_D, cfg.n_sink, lg)
+    mp = MlstmParams.for_head({k: v.numpy() for k, v in mw.items()}, h)
+    return prefill_mlstm(op, mp, Q, K, V, cfg.head_dim, G, prefill_override)
+
+
 def run_pair(cfg, weights, b: int, h: int, prompt_len: int, n_steps: int,
              prefill_override: Optional[np.ndarray] = None,
              step_override: Optional[Callable[[int], float]] = None,
-             attend: bool = True, layer: int = 0, keep_cache: bool = False) -> PairTrace:
-    """Prefill (b, h) with its prompt, then run ``n_steps`` decode steps."""
+             attend: bool = True, layer: int = 0, keep_cache: bool = False,
+             mlstm: Optional[dict] = None) -> PairTrace:
+    """Prefill (b, h) with its prompt, then run ``n_steps`` decode steps.
+
+    With ``mlstm`` (weights from ``workload.gen.mlstm_weights``) the scorer is the
+    stateful mLSTM instead of the MLP in ``weights``."""
     G = cfg.q_per_kv
-    cache = prefill_pair(cfg, weights, b, h, prompt_len, prefill_override, layer)
+    if mlstm is not None:
+        cache = prefill_pair_mlstm(cfg, mlstm, b, h, prompt_len, prefill_override)
+    else:
+        cache = prefill_pair(cfg, weights, b, h, prompt_len, prefill_override, layer)
     tr = PairTrace(b, h, prompt_len)
     if n_steps:
         q, k, v = gen.decode_inputs(cfg, [prompt_len], 0, n_steps, layer=layer, b0=b)

@@ -30,6 +30,8 @@ struct kvpop_cache {
   float* W1s = nullptr;                 // slice-major scorer weights for it
   float* b1s = nullptr;
   float* w2s = nullptr;
+  bool mlstm = false;                   // stateful mLSTM scorer instead of the MLP
+  MlstmDev md{};
   // staging for kvpop_decode_step_host
   void* stage_q = nullptr;
   void* stage_k = nullptr;
@@ -140,6 +142,17 @@ std::vector<StateBuf> state_buffers(kvpop_cache* c) {
   };
 }
 
+std::vector<StateBuf> all_state_buffers(kvpop_cache* c) {
+  std::vector<StateBuf> v = state_buffers(c);
+  if (c->mlstm) {
+    const size_t pairs = c->dm.pairs, d = c->dm.d;
+    v.push_back({c->md.C, pairs * d * (d / 2) * 4});
+    v.push_back({c->md.z, pairs * d * 4});
+    v.push_back({c->md.m, pairs * 4});
+  }
+  return v;
+}
+
 }  // namespace
 
 namespace kvpop {
@@ -166,13 +179,21 @@ void kvpop_debug_fail_alloc_after(int32_t n) { g_fail_after = n > 0 ? n : 0; }
 
 const char* kvpop_last_error(void) { return g_last_error; }
 
-kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
-                              cudaStream_t stream, kvpop_cache** out) {
+static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* sc,
+                               const kvpop_mlstm_scorer* ms, cudaStream_t stream, kvpop_cache** out) {
   if (!out) return KVPOP_ERR_INVALID_ARG;
   *out = nullptr;
+  if (!cfg_in) return KVPOP_ERR_INVALID_ARG;
+  kvpop_config cfgv = *cfg_in;
+  if (ms) cfgv.scorer_hidden = 4;            // unused by the mLSTM scorer
+  const kvpop_config* cfg = &cfgv;
   kvpop_status vs = validate(cfg);
   if (vs != KVPOP_OK) return vs;
-  if (!sc || !sc->W1 || !sc->b1 || !sc->w2 || !sc->b2) return KVPOP_ERR_INVALID_ARG;
+  if (sc && (!sc->W1 || !sc->b1 || !sc->w2 || !sc->b2)) return KVPOP_ERR_INVALID_ARG;
+  if (ms && (!ms->Wq || !ms->Wk || !ms->Wv || !ms->wi || !ms->wf || !ms->bi || !ms->bf || !ms->a ||
+             !ms->b))
+    return KVPOP_ERR_INVALID_ARG;
+  if (!sc && !ms) return KVPOP_ERR_INVALID_ARG;
 
   kvpop_cache* c = new (std::nothrow) kvpop_cache();
   if (!c) return KVPOP_ERR_OOM;
@@ -185,6 +206,8 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
   dm.pairs = dm.batch * dm.H;
   c->esz = cfg->kv_dtype == KVPOP_F32 ? 4 : 2;
   c->magic = kMagic;
+  c->mlstm = ms != nullptr;
+  if (c->mlstm && !mlstm_ok(dm)) { delete c; return KVPOP_ERR_INVALID_ARG; }
   NOTE(cudaGetDevice(&c->device));
 
   const size_t pairs = dm.pairs, B = dm.B, D = dm.D, d = dm.d, H = dm.H, F = dm.F, Fp = dm.Fp;
@@ -239,7 +262,21 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
     s = from_cuda(NOTE(tc_make_maps(c->st, dm, tc_map_ptr(c))));
   }
   if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest(dm)));
-  c->use_cluster = cluster_ingest_ok(dm);
+  const size_t hh = d / 2, NCm = mlstm_nc(dm.d);
+  if (s == KVPOP_OK && c->mlstm) {
+    MlstmDev& md = c->md;
+    md.NC = (int)NCm;
+    s = dev_alloc(c, &p, pairs * d * hh * 4); md.C = (float*)p;
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * 4); md.z = (float*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * 4); md.m = (float*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, H * 2 * d * NCm * 4); md.Wcat = (float*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, (4 * H + H * hh) * 4); md.bi = (float*)p; }
+    if (s == KVPOP_OK) {
+      md.bf = md.bi + H; md.b = md.bf + H; md.a = md.b + H;
+      s = from_cuda(NOTE(prepare_mlstm(dm)));
+    }
+  }
+  c->use_cluster = !c->mlstm && cluster_ingest_ok(dm);
   const size_t FS = cluster_ingest_fs(dm);
   if (s == KVPOP_OK && c->use_cluster) {
     s = dev_alloc(c, &p, (H * 8 * I * FS + 2 * H * 8 * FS) * 4);
@@ -258,13 +295,42 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
     c->st.W1 = W1; c->st.b1 = b1; c->st.w2 = w2; c->st.b2 = b2;
     // hidden units padded to Fp with zero weights: rows of F floats into rows of Fp
     cudaError_t e = NOTE(cudaMemsetAsync(w, 0, wbytes, stream));
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && sc)
       e = NOTE(cudaMemcpy2DAsync(W1, Fp * 4, sc->W1, F * 4, F * 4, H * I, cudaMemcpyDefault, stream));
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && sc)
       e = NOTE(cudaMemcpy2DAsync(b1, Fp * 4, sc->b1, F * 4, F * 4, H, cudaMemcpyDefault, stream));
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && sc)
       e = NOTE(cudaMemcpy2DAsync(w2, Fp * 4, sc->w2, F * 4, F * 4, H, cudaMemcpyDefault, stream));
-    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
+    if (e == cudaSuccess && sc) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
+    std::vector<float> minus_inf;
+    if (c->mlstm) {
+      // mLSTM weights: column blocks of Wcat [2d][NC] = [W_k | W_v | W_q | w_i | w_f | 0]
+      MlstmDev& md = c->md;
+      const size_t n2 = 2 * d;
+      if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(md.Wcat, 0, H * n2 * NCm * 4, stream));
+      const float* blocks[3] = {ms->Wk, ms->Wv, ms->Wq};
+      for (size_t h = 0; h < H && e == cudaSuccess; ++h) {
+        float* dst = md.Wcat + h * n2 * NCm;
+        for (int bidx = 0; bidx < 3 && e == cudaSuccess; ++bidx)
+          e = NOTE(cudaMemcpy2DAsync(dst + bidx * hh, NCm * 4, blocks[bidx] + h * n2 * hh, hh * 4,
+                                     hh * 4, n2, cudaMemcpyDefault, stream));
+        if (e == cudaSuccess)
+          e = NOTE(cudaMemcpy2DAsync(dst + 3 * hh, NCm * 4, ms->wi + h * n2, 4, 4, n2,
+                                     cudaMemcpyDefault, stream));
+        if (e == cudaSuccess)
+          e = NOTE(cudaMemcpy2DAsync(dst + 3 * hh + 1, NCm * 4, ms->wf + h * n2, 4, 4, n2,
+                                     cudaMemcpyDefault, stream));
+      }
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(md.bi, ms->bi, H * 4, cudaMemcpyDefault, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(md.bf, ms->bf, H * 4, cudaMemcpyDefault, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(md.b, ms->b, H * 4, cudaMemcpyDefault, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(md.a, ms->a, H * hh * 4, cudaMemcpyDefault, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(md.C, 0, pairs * d * hh * 4, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(md.z, 0, pairs * d * 4, stream));
+      minus_inf.assign(pairs, -INFINITY);
+      if (e == cudaSuccess)
+        e = NOTE(cudaMemcpyAsync(md.m, minus_inf.data(), pairs * 4, cudaMemcpyHostToDevice, stream));
+    }
     if (c->use_cluster) {
       // slice-major copy for the cluster kernel: slice r holds hidden units [r*FS, r*FS + FS)
       const size_t nW = (H * 8 * I * FS + 2 * H * 8 * FS) * 4;
@@ -285,8 +351,9 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
                                      cudaMemcpyDefault, stream));
         }
     }
-    if (e == cudaSuccess && sc->log_gamma) {
-      e = NOTE(cudaMemcpyAsync(lg, sc->log_gamma, H * 4, cudaMemcpyDefault, stream));
+    const float* lg_src = sc ? sc->log_gamma : ms->log_gamma;
+    if (e == cudaSuccess && lg_src) {
+      e = NOTE(cudaMemcpyAsync(lg, lg_src, H * 4, cudaMemcpyDefault, stream));
       c->st.log_gamma = lg;
       c->has_decay = true;
     } else {
@@ -316,6 +383,24 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc,
   return KVPOP_OK;
 }
 
+kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* sc, cudaStream_t stream,
+                              kvpop_cache** out) {
+  if (!sc) {
+    if (out) *out = nullptr;
+    return KVPOP_ERR_INVALID_ARG;
+  }
+  return init_cache(cfg, sc, nullptr, stream, out);
+}
+
+kvpop_status kvpop_init_cache_mlstm(const kvpop_config* cfg, const kvpop_mlstm_scorer* ms,
+                                    cudaStream_t stream, kvpop_cache** out) {
+  if (!ms) {
+    if (out) *out = nullptr;
+    return KVPOP_ERR_INVALID_ARG;
+  }
+  return init_cache(cfg, nullptr, ms, stream, out);
+}
+
 kvpop_status kvpop_free(kvpop_cache* c) {
   if (!c) return KVPOP_OK;
   if (c->magic != kMagic) return KVPOP_ERR_INVALID_ARG;
@@ -343,9 +428,12 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
     return KVPOP_ERR_ALIGN;
   const size_t pairs = (size_t)n_seq * c->dm.H;
   const size_t prio_bytes = pairs * (size_t)Pmax * 4;
+  // the mLSTM prefill also needs every prompt token's features (k~, v~, q~, gates)
+  const size_t feat_bytes = c->mlstm ? pairs * (size_t)Pmax * mlstm_nf(c->dm.d) * 4 : 0;
+  const size_t feat_off = ((prio_bytes + 255) & ~size_t(255)) + 256;
   void* tmp = nullptr;
   if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
-  cudaError_t e = NOTE(cudaMallocAsync(&tmp, prio_bytes + 256 + (size_t)n_seq * 4, stream));
+  cudaError_t e = NOTE(cudaMallocAsync(&tmp, feat_off + feat_bytes + 256, stream));
   if (e != cudaSuccess) {
     cudaGetLastError();
     return from_cuda(e);
@@ -353,8 +441,16 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
   float* prio = static_cast<float*>(tmp);
   int32_t* plen_dev = reinterpret_cast<int32_t*>(static_cast<char*>(tmp) + ((prio_bytes + 255) & ~size_t(255)));
   e = NOTE(cudaMemcpyAsync(plen_dev, plen_host, (size_t)n_seq * 4, cudaMemcpyHostToDevice, stream));
-  if (e == cudaSuccess)
+  if (e == cudaSuccess && c->mlstm) {
+    float* feat = reinterpret_cast<float*>(static_cast<char*>(tmp) + feat_off);
+    e = NOTE(launch_prefill_mlstm_scores(c->st, c->dm, c->md, K, V, plen_dev, first_seq, n_seq, Pmax,
+                                         override_, feat, prio, stream));
+    if (e == cudaSuccess)
+      e = NOTE(launch_prefill_select(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, prio,
+                                     stream));
+  } else if (e == cudaSuccess) {
     e = NOTE(launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream));
+  }
   // the host copy of the lengths must outlive the async copy
   if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   cudaError_t e2 = cudaFreeAsync(tmp, stream);
@@ -371,6 +467,9 @@ kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, c
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned4(override_) ||
       !aligned4(evict_info) || !aligned4(score_out))
     return KVPOP_ERR_ALIGN;
+  if (c->mlstm)
+    return poison_on(c, NOTE(launch_ingest_mlstm(c->st, c->dm, c->md, q, k, v, override_, evict_info,
+                                                 score_out, stream)));
   if (c->use_cluster)
     return poison_on(c, NOTE(launch_ingest_cluster(c->st, c->dm, c->W1s, c->b1s, c->w2s, q, k, v,
                                                    override_, evict_info, score_out, stream)));
@@ -435,7 +534,7 @@ kvpop_status kvpop_export_state(kvpop_cache* c, void* host_buf, size_t* bytes, c
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
   if (!bytes) return KVPOP_ERR_INVALID_ARG;
-  auto bufs = state_buffers(c);
+  auto bufs = all_state_buffers(c);
   size_t need = 4 * sizeof(uint64_t) + sizeof(kvpop_config);
   for (auto& b : bufs) need += b.bytes;
   if (!host_buf) { *bytes = need; return KVPOP_OK; }
@@ -465,7 +564,7 @@ kvpop_status kvpop_import_state(kvpop_cache* c, const void* host_buf, size_t byt
   std::memcpy(hdr, in, sizeof(hdr));
   kvpop_config cfg;
   std::memcpy(&cfg, in + sizeof(hdr), sizeof(cfg));
-  auto bufs = state_buffers(c);
+  auto bufs = all_state_buffers(c);
   size_t need = sizeof(hdr) + sizeof(kvpop_config);
   for (auto& b : bufs) need += b.bytes;
   if (hdr[0] != kMagic || hdr[1] != kStateVersion || hdr[2] != need || bytes < need ||

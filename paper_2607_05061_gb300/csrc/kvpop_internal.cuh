@@ -82,6 +82,34 @@ cudaError_t attend_config(const Dims& dm, AttendConfig* out);
 cudaError_t launch_attend(const State& st, const Dims& dm, const void* q, float* out,
                           int grid, cudaStream_t stream);
 
+// Stateful mLSTM scorer (device arrays of one cache).
+struct MlstmDev {
+  float* C;                    // [pairs][d][d/2]  stabilised matrix memory
+  float* z;                    // [pairs][d]       normaliser
+  float* m;                    // [pairs]          log-scale of the stabiliser
+  float* Wcat;                 // [H][2d][NC]      columns [W_k | W_v | W_q | w_i | w_f | 0]
+  float* bi;                   // [H]
+  float* bf;                   // [H]
+  float* a;                    // [H][d/2]
+  float* b;                    // [H]
+  int NC;
+};
+int mlstm_nc(int d);
+int mlstm_nf(int d);
+bool mlstm_ok(const Dims& dm);
+cudaError_t prepare_mlstm(const Dims& dm);
+cudaError_t launch_ingest_mlstm(const State& st, const Dims& dm, const MlstmDev& m, const void* q,
+                                const void* k, const void* v, const float* override_,
+                                int32_t* evict_info, float* score_out, cudaStream_t stream);
+cudaError_t launch_prefill_mlstm_scores(const State& st, const Dims& dm, const MlstmDev& m,
+                                        const void* K, const void* V, const int32_t* plen,
+                                        int first_seq, int n_seq, int Pmax, const float* override_,
+                                        float* feat, float* prio, cudaStream_t stream);
+// Selection + compaction + window fill of the prefill, from precomputed priorities.
+cudaError_t launch_prefill_select(const State& st, const Dims& dm, const void* Q, const void* K,
+                                  const void* V, const int32_t* plen, int first_seq, int n_seq,
+                                  int Pmax, const float* prio, cudaStream_t stream);
+
 // Tensor-core attention for bf16 K/V (TMA tensor maps over the K/V stores).
 size_t tc_maps_size();
 cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out);

@@ -361,6 +361,22 @@ static cudaError_t prefill_t(const State& st, const Dims& dm, const void* Q, con
   return cudaGetLastError();
 }
 
+cudaError_t launch_prefill_select(const State& st, const Dims& dm, const void* Q, const void* K,
+                                  const void* V, const int32_t* plen, int first_seq, int n_seq,
+                                  int Pmax, const float* prio, cudaStream_t stream) {
+  const int pairs = n_seq * dm.H;
+  if (dm.dtype == KVPOP_F32) {
+    SelectArgs<float> sel{st, dm, (const float*)Q, (const float*)K, (const float*)V, plen, prio,
+                          first_seq, Pmax};
+    prefill_select_kernel<float><<<pairs, NT2, 0, stream>>>(sel);
+  } else {
+    SelectArgs<bf16> sel{st, dm, (const bf16*)Q, (const bf16*)K, (const bf16*)V, plen, prio,
+                         first_seq, Pmax};
+    prefill_select_kernel<bf16><<<pairs, NT2, 0, stream>>>(sel);
+  }
+  return cudaGetLastError();
+}
+
 cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const void* K,
                            const void* V, const int32_t* plen_dev, int first_seq, int n_seq,
                            int Pmax, const float* override_, float* tmp_prio,

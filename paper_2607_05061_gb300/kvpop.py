@@ -39,10 +39,17 @@ class kvpop_scorer(ctypes.Structure):
                 ("log_gamma", c_void_p)]
 
 
+class kvpop_mlstm_scorer(ctypes.Structure):
+    _fields_ = [(n, c_void_p) for n in ("Wq", "Wk", "Wv", "wi", "wf", "bi", "bf", "a", "b",
+                                        "log_gamma")]
+
+
 _P = c_void_p
 _SIGS = {
     "kvpop_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "kvpop_init_cache": (ctypes.c_int, [POINTER(kvpop_config), POINTER(kvpop_scorer), _P, POINTER(_P)]),
+    "kvpop_init_cache_mlstm": (ctypes.c_int, [POINTER(kvpop_config), POINTER(kvpop_mlstm_scorer), _P,
+                                              POINTER(_P)]),
     "kvpop_free": (ctypes.c_int, [_P]),
     "kvpop_prefill_compress": (ctypes.c_int, [_P, _P, _P, _P, POINTER(c_int32), c_int32, c_int32,
                                               c_int32, _P, _P]),
@@ -105,17 +112,30 @@ class KVpopCache:
     """One attention layer's compressed KV cache (library-owned device state)."""
 
     def __init__(self, batch: int, n_kv_heads: int, q_per_kv: int, head_dim: int, budget_B: int,
-                 delay_D: int, scorer_hidden: int, kv_dtype, W1, b1, w2, b2, log_gamma=None,
-                 n_sink: int = 0, stream=None):
+                 delay_D: int, scorer_hidden: int, kv_dtype, W1=None, b1=None, w2=None, b2=None,
+                 log_gamma=None, n_sink: int = 0, stream=None, mlstm: Optional[dict] = None):
+        """MLP scorer from ``W1, b1, w2, b2``; or, with ``mlstm`` (a dict of ``Wq, Wk, Wv,
+        wi, wf, bi, bf, a, b`` and optionally ``log_gamma``), the stateful mLSTM scorer."""
         self.cfg = kvpop_config(batch, n_kv_heads, q_per_kv, head_dim, budget_B, delay_D, n_sink,
                                 scorer_hidden, dtype_code(kv_dtype))
-        keep = [t.contiguous().float() for t in (W1, b1, w2, b2)]
-        lg = None if log_gamma is None else log_gamma.contiguous().float()
-        sc = kvpop_scorer(*[t.data_ptr() for t in keep], None if lg is None else lg.data_ptr())
         h = _P()
-        _ck(kvpop_init_cache(ctypes.byref(self.cfg), ctypes.byref(sc), _stream(stream), ctypes.byref(h)),
-            "kvpop_init_cache")
+        if mlstm is not None:
+            names = ("Wq", "Wk", "Wv", "wi", "wf", "bi", "bf", "a", "b")
+            keep = {n: mlstm[n].contiguous().float() for n in names}
+            lg = mlstm.get("log_gamma")
+            lg = None if lg is None else lg.contiguous().float()
+            ms = kvpop_mlstm_scorer(*[keep[n].data_ptr() for n in names],
+                                    None if lg is None else lg.data_ptr())
+            _ck(kvpop_init_cache_mlstm(ctypes.byref(self.cfg), ctypes.byref(ms), _stream(stream),
+                                       ctypes.byref(h)), "kvpop_init_cache_mlstm")
+        else:
+            keep = [t.contiguous().float() for t in (W1, b1, w2, b2)]
+            lg = None if log_gamma is None else log_gamma.contiguous().float()
+            sc = kvpop_scorer(*[t.data_ptr() for t in keep], None if lg is None else lg.data_ptr())
+            _ck(kvpop_init_cache(ctypes.byref(self.cfg), ctypes.byref(sc), _stream(stream),
+                                 ctypes.byref(h)), "kvpop_init_cache")
         self.handle = h.value
+        self.mlstm = mlstm is not None
         self.batch, self.H, self.G, self.d = batch, n_kv_heads, q_per_kv, head_dim
 
     def prefill(self, Q, K, V, prompt_lens: Sequence[int], first_seq: int = 0, override=None,
@@ -196,11 +216,15 @@ def parse_state(blob: bytes, cfg: kvpop_config) -> dict:
               ("len", np.int32, (pairs,), 4), ("min_score", np.float32, (pairs,), 4),
               ("min_slot", np.int32, (pairs,), 4),
               ("blk_score", np.float32, (pairs, (B + 63) // 64), 4),
-              ("blk_slot", np.int32, (pairs, (B + 63) // 64), 4)]
+              ("blk_slot", np.int32, (pairs, (B + 63) // 64), 4),
+              ("mlstm_C", np.float32, (pairs, d, d // 2), 4), ("mlstm_z", np.float32, (pairs, d), 4),
+              ("mlstm_m", np.float32, (pairs,), 4)]
     off = 4 * 8 + ctypes.sizeof(kvpop_config)
     out = {}
     for name, dt, shape, sz in layout:
         n = int(np.prod(shape)) * sz
+        if name.startswith("mlstm_") and off + n > len(blob):
+            break                                   # MLP-scorer caches have no recurrent state
         out[name] = np.frombuffer(blob, dtype=dt, count=int(np.prod(shape)), offset=off).reshape(shape)
         off += n
     return out

@@ -15,8 +15,12 @@ TOL = {"f32": 1e-5, "bf16": 2e-2}      # attention max-abs tolerance per K/V dty
 STREAM_PREFILL_OV, STREAM_DECODE_OV = 30, 31
 
 
-def make_cache(cfg, weights):
+def make_cache(cfg, weights, mlstm=None):
     from paper_2607_05061_gb300 import kvpop
+    if mlstm is not None:
+        return kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
+                                cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, n_sink=cfg.n_sink,
+                                mlstm=mlstm)
     W1, b1, w2, b2, lg = weights
     return kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
                             cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
@@ -80,7 +84,7 @@ def gpu_decode(cache, cfg, lengths, nsteps, device, override=None,
 
 
 def oracle_pairs(cfg, weights, lengths, nsteps, pairs, prefill_override=None, decode_override=None,
-                 attend=True):
+                 attend=True, mlstm=None):
     """Oracle traces for the listed (b, h) pairs (injected scores given as CPU tensors)."""
     from oracle.run import run_pair
     traces = []
@@ -92,7 +96,7 @@ def oracle_pairs(cfg, weights, lengths, nsteps, pairs, prefill_override=None, de
             col = decode_override[:, bb, hh].numpy()
             dov = (lambda c: (lambda j: float(c[j])))(col)
         traces.append(run_pair(cfg, weights, bb, hh, P, nsteps, prefill_override=pov,
-                               step_override=dov, attend=attend, keep_cache=True))
+                               step_override=dov, attend=attend, keep_cache=True, mlstm=mlstm))
     return traces
 
 

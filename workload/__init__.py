@@ -17,4 +17,5 @@ from .gen import (  # noqa: F401
     stack_weights,
     prompt_hidden,
     decode_hidden,
+    mlstm_weights,
 )

@@ -32,6 +32,7 @@ LP = 1 << 20            # positions per (sequence, head) stream
 
 STREAM_K, STREAM_V, STREAM_Q = 1, 2, 3
 STREAM_W1, STREAM_W2 = 10, 11
+STREAM_MLSTM = 12
 STREAM_LEN, STREAM_OUTLIER = 20, 21
 STREAM_HIDDEN, STREAM_WPROJ, STREAM_DECODE_HIDDEN = 40, 50, 60
 LAYER_STRIDE = 1000     # stream offset between layers of a stack
@@ -277,4 +278,38 @@ def decode_hidden(cfg, lengths: Sequence[int], step0: int, nsteps: int, device="
     base = ((bs[None, :] * LP + L[None, :] + steps[:, None]) * hid).reshape(-1)
     out = torch.empty((nsteps, len(lengths), hid), dtype=torch.bfloat16, device=device)
     _rows(cfg.seed, STREAM_DECODE_HIDDEN, base, hid, out.view(-1, hid))
+    return out
+
+
+def mlstm_weights(cfg, layer: int = 0) -> dict:
+    """Random-init stateful mLSTM scorer per KV head (fp32, CPU tensors).
+
+    Xavier-normal W_q, W_k, W_v [H][2d][d/2] and a [H][d/2]; gate weights
+    w_i, w_f [H][2d] ~ N(0, 1/(2d)); b_i = 0 and b_f = 3 (a forget gate near 0.95,
+    i.e. a memory of a few dozen tokens); b = 0.
+    """
+    H, d = cfg.n_kv_heads, cfg.head_dim
+    n2, hh = 2 * d, d // 2
+    st = STREAM_MLSTM + layer * LAYER_STRIDE
+    out = {}
+    off = 0
+
+    def draw(shape, std):
+        nonlocal off
+        n = int(np.prod(shape))
+        v = normal_values(cfg.seed, st, torch.arange(off, off + n, dtype=torch.int64))
+        off += n
+        return (v * np.float32(std)).view(*shape).contiguous()
+    xav = np.sqrt(2.0 / (n2 + hh))
+    out["Wq"] = draw((H, n2, hh), xav)
+    out["Wk"] = draw((H, n2, hh), xav)
+    out["Wv"] = draw((H, n2, hh), xav)
+    out["wi"] = draw((H, n2), 1.0 / np.sqrt(n2))
+    out["wf"] = draw((H, n2), 1.0 / np.sqrt(n2))
+    out["a"] = draw((H, hh), np.sqrt(2.0 / (hh + 1)))
+    out["bi"] = torch.zeros(H)
+    out["bf"] = torch.full((H,), 3.0)
+    out["b"] = torch.zeros(H)
+    if cfg.log_gamma != 0.0:
+        out["log_gamma"] = torch.full((H,), float(cfg.log_gamma))
     return out
