@@ -140,6 +140,70 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* cache, const void* Q_dev, const
                                     int32_t first_seq, int32_t n_seq, int32_t Pmax,
                                     const float* score_override_dev, cudaStream_t stream);
 
+/* Prompt compression with outputs (App. C.1 mask, App. C.3): everything
+ * kvpop_prefill_compress does, plus the attention output of every prompt query
+ * under the running top-k mask
+ *   M[q,t] = t < s  or  q - t < D  or  (s <= t <= q - D and rank(t) <= tau_q)
+ * (causal, t <= q), where rank orders the prompt tokens by static priority
+ * (higher first, earlier position on ties; the last D tokens, which have no
+ * score yet, rank last) and tau_q is the rank of the min(B - s, |E(q)|)-th best
+ * token of E(q) = {s <= t <= q - D} (-1 while E(q) is empty).  At q = P - 1 the
+ * retained set is exactly the cache prompt compression leaves.
+ *   Y_dev    [n_seq][H*G][Pmax][d] fp32 out   (rows q >= P untouched)
+ *   lse_dev  [n_seq][H*G][Pmax] fp32 out, natural log of the softmax
+ *            normaliser over the retained keys (the sparse LSE of App. D.3),
+ *            or NULL
+ *   rank_dev, tau_dev [n_seq][H][Pmax] int32 out (-1 past P), or NULL
+ * Other arguments as kvpop_prefill_compress.  Needs Pmax <= 262144,
+ * n_seq*H <= 65535, d in {64, 128}, G in {1, 2, 4} and per-tile key lists of
+ * 4*(B + s + 2*128 + D) bytes that fit in shared memory (else
+ * KVPOP_ERR_INVALID_ARG).  bf16 runs on tensor cores, fp32 on CUDA cores.
+ * Temporaries: 24 bytes per (sequence, head, token) on top of the compression's. */
+kvpop_status kvpop_prefill_attend(kvpop_cache* cache, const void* Q_dev, const void* K_dev,
+                                  const void* V_dev, const int32_t* prompt_len_host,
+                                  int32_t first_seq, int32_t n_seq, int32_t Pmax,
+                                  const float* score_override_dev, float* Y_dev, float* lse_dev,
+                                  int32_t* rank_dev, int32_t* tau_dev, cudaStream_t stream);
+
+/* Bytes of device workspace kvpop_topk_cutoff needs (0 for an empty problem). */
+size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S);
+
+/* Running top-k cutoffs of n_rows independent rows (App. C.1 ranks, App. C.2 /
+ * Algorithm 2 cutoffs), no cache involved.  Row r holds lengths_dev[r] tokens
+ * (S for every row if lengths_dev is NULL) with fp32 static priorities
+ * prio_dev[r][t] (NaN counts as -inf, -0 as +0).  Outputs:
+ *   rank_dev [n_rows][S]  rank of token t: 0 = highest priority, equal
+ *                         priorities by position; -1 past the row length
+ *   tau_dev  [n_rows][S]  rank of the min(k, |E(q)|)-th best token of
+ *                         E(q) = {n_sink <= t <= q - window}; -1 while E(q) is
+ *                         empty and past the row length
+ * Where Algorithm 2 leaves tau_q = -1 while fewer than k tokens are eligible,
+ * this keeps all of them (the top k of a set smaller than k is the set).
+ * workspace_dev: kvpop_topk_workspace_bytes(n_rows, S) bytes, 256-byte aligned,
+ * owned by the caller.  S <= 262144, window >= 1, k >= 1.  Asynchronous on
+ * `stream`; no allocation. */
+kvpop_status kvpop_topk_cutoff(const float* prio_dev, const int32_t* lengths_dev, int32_t n_rows,
+                               int32_t S, int32_t n_sink, int32_t window, int32_t k,
+                               int32_t* rank_dev, int32_t* tau_dev, void* workspace_dev,
+                               size_t workspace_bytes, cudaStream_t stream);
+
+/* Masked causal attention over prompts under the running top-k mask given by
+ * rank / tau from kvpop_topk_cutoff (same n_sink, window and k), no cache
+ * involved.  Per KV head h and query head g = 0..G-1:
+ *   y[q] = sum_t softmax_t(M[q,t] ? q.k_t / sqrt(d) : -inf) v_t
+ *   Q_dev [n_seq][H*G][S][d], K_dev, V_dev [n_seq][H][S][d]  (dtype)
+ *   rank_dev, tau_dev [n_seq][H][S] int32;  lengths_dev [n_seq] or NULL (= S)
+ *   Y_dev [n_seq][H*G][S][d] fp32 out; lse_dev [n_seq][H*G][S] fp32 out or NULL
+ * Limits as kvpop_prefill_attend.  Asynchronous on `stream`; no allocation.
+ * rank / tau that did not come from kvpop_topk_cutoff give unspecified outputs
+ * but never an out-of-bounds access. */
+kvpop_status kvpop_prompt_attention(const void* Q_dev, const void* K_dev, const void* V_dev,
+                                    const int32_t* rank_dev, const int32_t* tau_dev,
+                                    const int32_t* lengths_dev, int32_t n_seq, int32_t n_kv_heads,
+                                    int32_t q_per_kv, int32_t head_dim, int32_t S, int32_t n_sink,
+                                    int32_t window, int32_t k, kvpop_dtype dtype, float* Y_dev,
+                                    float* lse_dev, cudaStream_t stream);
+
 /* Decode steps 1-4 for every sequence: ingest the token at position p = len,
  * score u = p - D (if p >= D), keep or drop it, scatter it, push p.
  *   q_dev [b][H*G][d], k_dev / v_dev [b][H][d]

@@ -412,9 +412,14 @@ kvpop_status kvpop_free(kvpop_cache* c) {
   return KVPOP_OK;
 }
 
-kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K, const void* V,
-                                    const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
-                                    int32_t Pmax, const float* override_, cudaStream_t stream) {
+namespace {
+
+// Prompt compression, optionally with the prompt's attention outputs under the
+// running top-k mask (Y != nullptr).
+kvpop_status prefill_impl(kvpop_cache* c, const void* Q, const void* K, const void* V,
+                          const int32_t* plen_host, int32_t first_seq, int32_t n_seq, int32_t Pmax,
+                          const float* override_, float* Y, float* lse, int32_t* rank_out,
+                          int32_t* tau_out, cudaStream_t stream) {
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
   if (!plen_host || n_seq < 0 || first_seq < 0 || first_seq + (long long)n_seq > c->dm.batch ||
@@ -426,23 +431,38 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
   if (Pmax > 0 && (!Q || !K || !V)) return KVPOP_ERR_INVALID_ARG;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned4(override_))
     return KVPOP_ERR_ALIGN;
+  const bool outputs = Y != nullptr;
+  if (outputs) {
+    if (!aligned16(Y) || !aligned4(lse) || !aligned4(rank_out) || !aligned4(tau_out))
+      return KVPOP_ERR_ALIGN;
+    if (Pmax > kTopkMaxS || (long long)n_seq * c->dm.H > 65535 ||
+        !prompt_attend_ok(c->dm.dtype, c->dm.d, c->dm.G, c->dm.s, c->dm.D, c->dm.B - c->dm.s))
+      return KVPOP_ERR_INVALID_ARG;
+  }
   const size_t pairs = (size_t)n_seq * c->dm.H;
-  const size_t prio_bytes = pairs * (size_t)Pmax * 4;
+  auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+  const size_t prio_bytes = al(pairs * (size_t)Pmax * 4);
   // the mLSTM prefill also needs every prompt token's features (k~, v~, q~, gates)
   const size_t feat_bytes = c->mlstm ? pairs * (size_t)Pmax * mlstm_nf(c->dm.d) * 4 : 0;
-  const size_t feat_off = ((prio_bytes + 255) & ~size_t(255)) + 256;
+  const size_t plen_off = prio_bytes;
+  const size_t feat_off = plen_off + 256;
+  const size_t rank_off = al(feat_off + feat_bytes);
+  const size_t tau_off = rank_off + (outputs && !rank_out ? prio_bytes : 0);
+  const size_t ws_off = tau_off + (outputs && !tau_out ? prio_bytes : 0);
+  const size_t ws_bytes = outputs ? topk_workspace_bytes((int)pairs, Pmax) : 0;
   void* tmp = nullptr;
   if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
-  cudaError_t e = NOTE(cudaMallocAsync(&tmp, feat_off + feat_bytes + 256, stream));
+  cudaError_t e = NOTE(cudaMallocAsync(&tmp, ws_off + ws_bytes + 256, stream));
   if (e != cudaSuccess) {
     cudaGetLastError();
     return from_cuda(e);
   }
-  float* prio = static_cast<float*>(tmp);
-  int32_t* plen_dev = reinterpret_cast<int32_t*>(static_cast<char*>(tmp) + ((prio_bytes + 255) & ~size_t(255)));
+  char* base = static_cast<char*>(tmp);
+  float* prio = reinterpret_cast<float*>(base);
+  int32_t* plen_dev = reinterpret_cast<int32_t*>(base + plen_off);
   e = NOTE(cudaMemcpyAsync(plen_dev, plen_host, (size_t)n_seq * 4, cudaMemcpyHostToDevice, stream));
   if (e == cudaSuccess && c->mlstm) {
-    float* feat = reinterpret_cast<float*>(static_cast<char*>(tmp) + feat_off);
+    float* feat = reinterpret_cast<float*>(base + feat_off);
     e = NOTE(launch_prefill_mlstm_scores(c->st, c->dm, c->md, K, V, plen_dev, first_seq, n_seq, Pmax,
                                          override_, feat, prio, stream));
     if (e == cudaSuccess)
@@ -451,11 +471,80 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
   } else if (e == cudaSuccess) {
     e = NOTE(launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream));
   }
+  if (e == cudaSuccess && outputs && Pmax > 0) {
+    int32_t* rank = rank_out ? rank_out : reinterpret_cast<int32_t*>(base + rank_off);
+    int32_t* tau = tau_out ? tau_out : reinterpret_cast<int32_t*>(base + tau_off);
+    const int s_ = c->dm.s, D = c->dm.D, k = c->dm.B - c->dm.s;
+    e = NOTE(launch_topk(prio, plen_dev, c->dm.H, D, (int)pairs, Pmax, s_, D, k, rank, tau,
+                         base + ws_off, stream));
+    if (e == cudaSuccess)
+      e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, plen_dev, n_seq, c->dm.H, c->dm.G, c->dm.d,
+                                    Pmax, s_, D, k, c->dm.dtype, Y, lse, c->st.err, stream));
+  }
   // the host copy of the lengths must outlive the async copy
   if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   cudaError_t e2 = cudaFreeAsync(tmp, stream);
   if (e == cudaSuccess) e = e2;
   return poison_on(c, e);
+}
+
+}  // namespace
+
+kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K, const void* V,
+                                    const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
+                                    int32_t Pmax, const float* override_, cudaStream_t stream) {
+  return prefill_impl(c, Q, K, V, plen_host, first_seq, n_seq, Pmax, override_, nullptr, nullptr,
+                      nullptr, nullptr, stream);
+}
+
+kvpop_status kvpop_prefill_attend(kvpop_cache* c, const void* Q, const void* K, const void* V,
+                                  const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
+                                  int32_t Pmax, const float* override_, float* Y, float* lse,
+                                  int32_t* rank_out, int32_t* tau_out, cudaStream_t stream) {
+  if (!Y) return KVPOP_ERR_INVALID_ARG;
+  return prefill_impl(c, Q, K, V, plen_host, first_seq, n_seq, Pmax, override_, Y, lse, rank_out,
+                      tau_out, stream);
+}
+
+size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S) {
+  if (n_rows <= 0 || S <= 0) return 0;
+  return topk_workspace_bytes(n_rows, S);
+}
+
+kvpop_status kvpop_topk_cutoff(const float* prio, const int32_t* lengths, int32_t n_rows, int32_t S,
+                               int32_t n_sink, int32_t window, int32_t k, int32_t* rank, int32_t* tau,
+                               void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  if (n_rows < 0 || S < 0 || S > kTopkMaxS || n_sink < 0 || window < 1 || k < 1)
+    return KVPOP_ERR_INVALID_ARG;
+  if (n_rows == 0 || S == 0) return KVPOP_OK;
+  if (!prio || !rank || !tau || !workspace) return KVPOP_ERR_INVALID_ARG;
+  if (workspace_bytes < topk_workspace_bytes(n_rows, S)) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned4(prio) || !aligned4(lengths) || !aligned4(rank) || !aligned4(tau) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return KVPOP_ERR_ALIGN;
+  cudaError_t e = NOTE(launch_topk(prio, lengths, 1, 0, n_rows, S, n_sink, window, k, rank, tau,
+                                   workspace, stream));
+  return from_cuda(e);
+}
+
+kvpop_status kvpop_prompt_attention(const void* Q, const void* K, const void* V, const int32_t* rank,
+                                    const int32_t* tau, const int32_t* lengths, int32_t n_seq,
+                                    int32_t n_kv_heads, int32_t q_per_kv, int32_t head_dim, int32_t S,
+                                    int32_t n_sink, int32_t window, int32_t k, kvpop_dtype dtype,
+                                    float* Y, float* lse, cudaStream_t stream) {
+  if (n_seq < 0 || n_kv_heads < 1 || S < 0 || n_sink < 0 || window < 1 || k < 1 ||
+      (dtype != KVPOP_F32 && dtype != KVPOP_BF16) || (long long)n_seq * n_kv_heads > 65535 ||
+      !prompt_attend_ok(dtype, head_dim, q_per_kv, n_sink, window, k))
+    return KVPOP_ERR_INVALID_ARG;
+  if (n_seq == 0 || S == 0) return KVPOP_OK;
+  if (!Q || !K || !V || !rank || !tau || !Y) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(Y) || !aligned4(rank) ||
+      !aligned4(tau) || !aligned4(lengths) || !aligned4(lse))
+    return KVPOP_ERR_ALIGN;
+  cudaError_t e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, lengths, n_seq, n_kv_heads, q_per_kv,
+                                            head_dim, S, n_sink, window, k, dtype, Y, lse, nullptr,
+                                            stream));
+  return from_cuda(e);
 }
 
 kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, const void* v,

@@ -122,6 +122,21 @@ cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const
                            int Pmax, const float* override_, float* tmp_prio,
                            cudaStream_t stream);
 
+// Running top-k over a prompt (App. C): static ranks and per-query cutoffs of
+// n_rows rows of S tokens; row r has len[r / rows_per_len] tokens (S if len is
+// null), the last `tail` of them without a priority.
+constexpr int kTopkMaxS = 1 << 18;
+size_t topk_workspace_bytes(int n_rows, int S);
+cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len, int tail,
+                        int n_rows, int S, int s, int w, int k, int32_t* rank, int32_t* tau,
+                        void* workspace, cudaStream_t stream);
+// Masked causal attention over a prompt under the running top-k mask.
+bool prompt_attend_ok(int dtype, int d, int G, int s, int w, int k);
+cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, const int32_t* rank,
+                                 const int32_t* tau, const int32_t* len, int n_seq, int H, int G,
+                                 int d, int S, int s, int w, int k, int dtype, float* Y, float* lse,
+                                 int32_t* err, cudaStream_t stream);
+
 // ------------------------------------------------------------------ device helpers
 __device__ __forceinline__ float to_f(float x) { return x; }
 __device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }

@@ -83,3 +83,37 @@ def test_free_null_and_foreign_handles(kv):
 def test_alloc_fault_hook_is_callable(kv):
     kv.kvpop_debug_fail_alloc_after(0)
     kv.kvpop_debug_fail_alloc_after(-5)
+
+
+def test_topk_and_prompt_attention_reject_bad_arguments(kv):
+    """Argument checks of the cache-free prompt calls run before any CUDA call."""
+    P = 0x1000                                   # 16-byte aligned dummy address, never dereferenced
+    ws = kv.kvpop_topk_workspace_bytes(4, 100)
+    assert ws >= 4 * 100 * 16
+    assert kv.kvpop_topk_workspace_bytes(0, 100) == 0
+    ok, bad, align = 0, 1, 2          # KVPOP_OK, KVPOP_ERR_INVALID_ARG, KVPOP_ERR_ALIGN
+    cut = kv.kvpop_topk_cutoff
+    assert cut(P, None, 0, 100, 0, 4, 8, P, P, P, ws, None) == ok          # nothing to do
+    assert cut(P, None, 4, 100, 0, 0, 8, P, P, P, ws, None) == bad         # window 0
+    assert cut(P, None, 4, 100, 0, 4, 0, P, P, P, ws, None) == bad         # k 0
+    assert cut(P, None, 4, (1 << 18) + 1, 0, 4, 8, P, P, P, ws, None) == bad
+    assert cut(P, None, 4, 100, 0, 4, 8, P, P, P, ws - 1, None) == bad     # workspace too small
+    assert cut(None, None, 4, 100, 0, 4, 8, P, P, P, ws, None) == bad
+    assert cut(P + 2, None, 4, 100, 0, 4, 8, P, P, P, ws, None) == align
+    assert cut(P, None, 4, 100, 0, 4, 8, P, P, P + 16, ws, None) == align  # workspace 256-aligned
+    att = kv.kvpop_prompt_attention
+    args = lambda **o: [o.get(n, v) for n, v in (
+        ("Q", P), ("K", P), ("V", P), ("rank", P), ("tau", P), ("len", None), ("n", 2), ("H", 8),
+        ("G", 4), ("d", 128), ("S", 64), ("s", 0), ("w", 16), ("k", 64), ("dt", kv.KVPOP_BF16),
+        ("Y", P), ("lse", P), ("st", None))]
+    assert att(*args(n=0)) == ok
+    assert att(*args(d=96)) == bad
+    assert att(*args(G=3)) == bad
+    assert att(*args(w=0)) == bad
+    assert att(*args(k=1 << 20)) == bad                 # key lists would not fit in shared memory
+    assert att(*args(n=10000)) == bad                   # more than 65535 (sequence, head) rows
+    assert att(*args(dt=7)) == bad
+    assert att(*args(Y=None)) == bad
+    assert att(*args(Q=P + 8)) == align
+    assert att(*args(Y=P + 4)) == align
+    assert att(*args(lse=P + 2)) == align
