@@ -204,6 +204,39 @@ kvpop_status kvpop_prompt_attention(const void* Q_dev, const void* K_dev, const 
                                     int32_t window, int32_t k, kvpop_dtype dtype, float* Y_dev,
                                     float* lse_dev, cudaStream_t stream);
 
+/* Dense causal log-normalisers (App. D.1), the exact-target variant of the
+ * normaliser fed to kvpop_future_target:
+ *   lse[q] = log sum_{t <= q} exp(q.k_t / sqrt(d))   per query head, natural log
+ *   Q_dev [n_seq][H*G][S][d], K_dev [n_seq][H][S][d] (dtype); lengths_dev [n_seq]
+ *   or NULL (= S); lse_dev [n_seq][H*G][S] fp32 out (rows past a length untouched)
+ * d in {64, 128}, G in {1, 2, 4}, n_seq*H <= 65535.  Asynchronous; no allocation. */
+kvpop_status kvpop_causal_lse(const void* Q_dev, const void* K_dev, const int32_t* lengths_dev,
+                              int32_t n_seq, int32_t n_kv_heads, int32_t q_per_kv,
+                              int32_t head_dim, int32_t S, kvpop_dtype dtype, float* lse_dev,
+                              cudaStream_t stream);
+
+/* Future-attention target for training the scorer (Sec. 3.4, App. D, App. F).
+ * Transposed attention pass (App. D.2), for every key t and query head g:
+ *   logm[g][t] = log sum_{d = t+w}^{hi} exp(q_d.k_t / sqrt(d) - lse_dev[g][d])
+ * with hi = S_b - 1, or min(S_b - 1, t + w + lookahead) when lookahead > 0
+ * (-inf when the range is empty).  lse_dev is the dense normaliser of
+ * kvpop_causal_lse (exact target) or the sparse one of kvpop_prompt_attention /
+ * kvpop_prefill_attend (approximate target, App. D.3).  If target_dev is not
+ * NULL it also receives, per KV head (Eq. 2, App. F.1-F.2),
+ *   target[t] = log(eps + Agg_g exp(logm[g][t]) / N_t),
+ *   Agg = max (agg 0) or mean (agg 1), N_t = max(1, S_b - (t + w)) clipped to
+ *   lookahead + 1 when lookahead > 0, N_t = 1 when count_norm is 0.
+ *   Q_dev [n_seq][H*G][S][d], K_dev [n_seq][H][S][d]; lse_dev, logm_dev
+ *   [n_seq][H*G][S] fp32; target_dev [n_seq][H][S] fp32; lengths_dev [n_seq] or
+ *   NULL (S_b = S).  window >= 0, lookahead >= 0, eps >= 0 finite.
+ * Asynchronous on `stream`; no allocation. */
+kvpop_status kvpop_future_target(const void* Q_dev, const void* K_dev, const float* lse_dev,
+                                 const int32_t* lengths_dev, int32_t n_seq, int32_t n_kv_heads,
+                                 int32_t q_per_kv, int32_t head_dim, int32_t S, int32_t window,
+                                 int32_t lookahead, kvpop_dtype dtype, float* logm_dev,
+                                 float* target_dev, int32_t agg, int32_t count_norm, float eps,
+                                 cudaStream_t stream);
+
 /* Decode steps 1-4 for every sequence: ingest the token at position p = len,
  * score u = p - D (if p >= D), keep or drop it, scatter it, push p.
  *   q_dev [b][H*G][d], k_dev / v_dev [b][H][d]

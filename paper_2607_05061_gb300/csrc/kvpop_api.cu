@@ -547,6 +547,39 @@ kvpop_status kvpop_prompt_attention(const void* Q, const void* K, const void* V,
   return from_cuda(e);
 }
 
+kvpop_status kvpop_causal_lse(const void* Q, const void* K, const int32_t* lengths, int32_t n_seq,
+                              int32_t n_kv_heads, int32_t q_per_kv, int32_t head_dim, int32_t S,
+                              kvpop_dtype dtype, float* lse, cudaStream_t stream) {
+  if (n_seq < 0 || n_kv_heads < 1 || S < 0 || (dtype != KVPOP_F32 && dtype != KVPOP_BF16) ||
+      (long long)n_seq * n_kv_heads > 65535 || !prompt_attend_ok(dtype, head_dim, q_per_kv, 0, 1, 1))
+    return KVPOP_ERR_INVALID_ARG;
+  if (n_seq == 0 || S == 0) return KVPOP_OK;
+  if (!Q || !K || !lse) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned4(lse) || !aligned4(lengths)) return KVPOP_ERR_ALIGN;
+  return from_cuda(NOTE(launch_causal_lse(Q, K, lengths, n_seq, n_kv_heads, q_per_kv, head_dim, S,
+                                          dtype, lse, stream)));
+}
+
+kvpop_status kvpop_future_target(const void* Q, const void* K, const float* lse,
+                                 const int32_t* lengths, int32_t n_seq, int32_t n_kv_heads,
+                                 int32_t q_per_kv, int32_t head_dim, int32_t S, int32_t window,
+                                 int32_t lookahead, kvpop_dtype dtype, float* logm, float* target,
+                                 int32_t agg, int32_t count_norm, float eps, cudaStream_t stream) {
+  if (n_seq < 0 || n_kv_heads < 1 || S < 0 || window < 0 || lookahead < 0 ||
+      (dtype != KVPOP_F32 && dtype != KVPOP_BF16) || (long long)n_seq * n_kv_heads > 65535 ||
+      !prompt_attend_ok(dtype, head_dim, q_per_kv, 0, 1, 1) || (agg != 0 && agg != 1) ||
+      (count_norm != 0 && count_norm != 1) || !(eps >= 0.f) || eps == INFINITY)
+    return KVPOP_ERR_INVALID_ARG;
+  if (n_seq == 0 || S == 0) return KVPOP_OK;
+  if (!Q || !K || !lse || !logm) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned4(lse) || !aligned4(lengths) || !aligned4(logm) ||
+      !aligned4(target))
+    return KVPOP_ERR_ALIGN;
+  return from_cuda(NOTE(launch_future_target(Q, K, lse, lengths, n_seq, n_kv_heads, q_per_kv,
+                                             head_dim, S, window, lookahead, dtype, logm, target,
+                                             agg, count_norm, eps, stream)));
+}
+
 kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, const void* v,
                                  const float* override_, int32_t* evict_info, float* score_out,
                                  cudaStream_t stream) {

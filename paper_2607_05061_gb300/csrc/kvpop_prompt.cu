@@ -24,7 +24,7 @@
 // fp32: CUDA-core kernel, one warp per (query, head) row, 32 keys per round.
 #include <climits>
 
-#include "kvpop_internal.cuh"
+#include "kvpop_mma.cuh"
 
 namespace kvpop {
 namespace {
@@ -71,7 +71,7 @@ __device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int
   ti.seq = ti.pair / a.H;
   ti.h = ti.pair - ti.seq * a.H;
   ti.L = a.len ? max(0, min(a.len[ti.seq], a.S)) : a.S;
-  ti.q0 = blockIdx.x * BM;
+  ti.q0 = (gridDim.x - 1 - blockIdx.x) * BM;        // longest tiles first
   if (ti.q0 >= ti.L) return false;
   ti.q1 = min(ti.q0 + BM - 1, ti.L - 1);
   const int nq = ti.q1 - ti.q0 + 1;
@@ -170,11 +170,27 @@ __device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int
   return true;
 }
 
+// Dense causal tiles (no mask beyond causality): keys 0 .. q0 serve every query
+// of the tile (list A), q0 + 1 .. q1 only the later ones (list M); a key's
+// list index is its position.
+__device__ __forceinline__ bool dense_setup(const PromptArgs& a, int BM, TileInfo& ti) {
+  ti.pair = blockIdx.y;
+  ti.seq = ti.pair / a.H;
+  ti.h = ti.pair - ti.seq * a.H;
+  ti.L = a.len ? max(0, min(a.len[ti.seq], a.S)) : a.S;
+  ti.q0 = (gridDim.x - 1 - blockIdx.x) * BM;
+  if (ti.q0 >= ti.L) return false;
+  ti.q1 = min(ti.q0 + BM - 1, ti.L - 1);
+  ti.nA = ti.q0 + 1;
+  ti.nM = ti.q1 - ti.q0;
+  return true;
+}
+
 // ---------------------------------------------------------------- CUDA-core kernel
 constexpr int SIMT_NT = 256;
 constexpr int SIMT_BM = 32;
 
-template <typename T, int HD>
+template <typename T, int HD, bool DENSE>
 __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
   extern __shared__ __align__(16) unsigned char smem_simt[];
   unsigned char* smem = smem_simt;
@@ -186,13 +202,18 @@ __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
   int32_t* posA = red + NW + 2;
   int32_t* posM = posA + a.capA;
   TileInfo ti;
-  if (!tile_setup<SIMT_NT>(a, SIMT_BM, tauS, red, posA, posM, ti)) return;
+  if (DENSE) {
+    if (!dense_setup(a, SIMT_BM, ti)) return;
+  } else if (!tile_setup<SIMT_NT>(a, SIMT_BM, tauS, red, posA, posM, ti)) {
+    return;
+  }
+  const bool want_y = a.Y != nullptr;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int G = a.G, H = a.H, S = a.S;
   const int nA = ti.nA, nU = ti.nA + ti.nM;
   const T* Kp = static_cast<const T*>(a.K) + (size_t)ti.pair * S * HD;
   const T* Vp = static_cast<const T*>(a.V) + (size_t)ti.pair * S * HD;
-  const int32_t* rank = a.rank + (size_t)ti.pair * S;
+  const int32_t* rank = DENSE ? nullptr : a.rank + (size_t)ti.pair * S;
   float* q_s = qv + warp * HD;
   for (int r = warp; r < SIMT_BM * G; r += NW) {
     const int ql = r / G, g = r - ql * G, q = ti.q0 + ql;
@@ -201,7 +222,7 @@ __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
     const T* qp = static_cast<const T*>(a.Q) + row * HD;
     for (int i = lane; i < HD; i += 32) q_s[i] = to_f(qp[i]) * a.qscale;
     __syncwarp();
-    const int tq = tauS[ql];
+    const int tq = DENSE ? 0 : tauS[ql];
     float m = -INFINITY, l = 0.f, o[NC];
 #pragma unroll
     for (int c = 0; c < NC; ++c) o[c] = 0.f;
@@ -210,8 +231,13 @@ __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
       int t = 0;
       bool keep = false;
       if (e < nU) {
-        t = e < nA ? posA[e] : posM[e - nA];
-        keep = e < nA || keep_key(q, t, __ldg(rank + t), tq, a.s, a.w);
+        if (DENSE) {
+          t = e;
+          keep = t <= q;
+        } else {
+          t = e < nA ? posA[e] : posM[e - nA];
+          keep = e < nA || keep_key(q, t, __ldg(rank + t), tq, a.s, a.w);
+        }
       }
       float logit = -INFINITY;
       if (keep) {
@@ -232,6 +258,8 @@ __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
 #pragma unroll
       for (int o2 = 16; o2; o2 >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o2);
       l = l * alpha + ps;
+      m = m_new;
+      if (!want_y) continue;
 #pragma unroll
       for (int c = 0; c < NC; ++c) o[c] *= alpha;
       const int nk = min(32, nU - e0);
@@ -244,60 +272,19 @@ __global__ void __launch_bounds__(SIMT_NT) prompt_simt_kernel(PromptArgs a) {
           for (int c = 0; c < NC; ++c) o[c] = fmaf(pj, to_f(vr[lane + 32 * c]), o[c]);
         }
       }
-      m = m_new;
     }
-    const float inv = 1.f / l;
-    float* yp = a.Y + row * HD;
+    if (want_y) {
+      const float inv = 1.f / l;
+      float* yp = a.Y + row * HD;
 #pragma unroll
-    for (int c = 0; c < NC; ++c) yp[lane + 32 * c] = o[c] * inv;
+      for (int c = 0; c < NC; ++c) yp[lane + 32 * c] = o[c] * inv;
+    }
     if (a.lse && lane == 0) a.lse[row] = (m + log2f(l)) * kLn2;
     __syncwarp();
   }
 }
 
 // ---------------------------------------------------------------- tensor-core kernel
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a0, uint32_t& a1, uint32_t& a2,
-                                        uint32_t& a3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& a0, uint32_t& a1, uint32_t& a2,
-                                          uint32_t& a3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
-                                         uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7},"
-      " {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
 template <int HD, int G>
 struct TcP {
   static constexpr int NW = 8;
@@ -321,11 +308,7 @@ struct TcP {
   static_assert(ROWS * ROWB <= STAGE, "the Q tile is staged in the first K/V stage");
 };
 
-__device__ __forceinline__ uint32_t swz(int row, int chunk, int rowb) {
-  return (uint32_t)(row * rowb + ((chunk ^ (row & 7)) << 4));
-}
-
-template <int HD, int G>
+template <int HD, int G, bool DENSE, bool WANT_Y>
 __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(PromptArgs a) {
   using P = TcP<HD, G>;
   extern __shared__ __align__(1024) unsigned char smem_tc[];
@@ -337,14 +320,18 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
   int32_t* posA = reinterpret_cast<int32_t*>(smem + P::OFF_LIST);
   int32_t* posM = posA + a.capA;
   TileInfo ti;
-  if (!tile_setup<P::THREADS>(a, P::BM, tauS, red, posA, posM, ti)) return;
+  if (DENSE) {
+    if (!dense_setup(a, P::BM, ti)) return;
+  } else if (!tile_setup<P::THREADS>(a, P::BM, tauS, red, posA, posM, ti)) {
+    return;
+  }
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int H = a.H, S = a.S;
   const int nA = ti.nA, nU = ti.nA + ti.nM;
   const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(smem);
   const bf16* Kp = static_cast<const bf16*>(a.K) + (size_t)ti.pair * S * HD;
-  const bf16* Vp = static_cast<const bf16*>(a.V) + (size_t)ti.pair * S * HD;
-  const int32_t* rank = a.rank + (size_t)ti.pair * S;
+  const bf16* Vp = WANT_Y ? static_cast<const bf16*>(a.V) + (size_t)ti.pair * S * HD : nullptr;
+  const int32_t* rank = DENSE ? nullptr : a.rank + (size_t)ti.pair * S;
   const bf16* Qbase = static_cast<const bf16*>(a.Q) + ((size_t)ti.seq * H * G + (size_t)ti.h * G) * S * HD;
 
   // Q tile -> stage 0 (rows past the prompt are zero-filled)
@@ -367,29 +354,33 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
   }
   __syncthreads();
 
-  const int pad_t = nA > 0 ? posA[0] : posM[0];
+  const int pad_t = DENSE ? 0 : (nA > 0 ? posA[0] : posM[0]);
+  // position of list entry e (entries past the list gather a valid row and are masked)
+  auto entry = [&](int e) {
+    if (DENSE) return e < nU ? e : pad_t;
+    return e < nA ? posA[e] : (e < nU ? posM[e - nA] : pad_t);
+  };
   auto issue = [&](int blk, int st) {
     const uint32_t kdst = sbase + st * P::STAGE;
     const uint32_t vdst = kdst + P::KVB;
     for (int i = tid; i < P::BN * P::CH; i += P::THREADS) {
       const int key = i / P::CH, c = i - key * P::CH;
-      const int e = blk * P::BN + key;
-      const int t = e < nA ? posA[e] : (e < nU ? posM[e - nA] : pad_t);
+      const int t = entry(blk * P::BN + key);
       const uint32_t off = swz(key, c, P::ROWB);
       cp_async16(kdst + off, Kp + (size_t)t * HD + c * 8, 16);
-      cp_async16(vdst + off, Vp + (size_t)t * HD + c * 8, 16);
+      if (WANT_Y) cp_async16(vdst + off, Vp + (size_t)t * HD + c * 8, 16);
     }
     if (tid < P::BN) {
       const int e = blk * P::BN + tid;
-      const int t = e < nA ? posA[e] : (e < nU ? posM[e - nA] : pad_t);
+      const int t = entry(e);
       posb[st * P::BN + tid] = e < nU ? t : INT_MAX;
-      cp_async4(sbase + P::OFF_RKB + (st * P::BN + tid) * 4, rank + t);
+      if (!DENSE) cp_async4(sbase + P::OFF_RKB + (st * P::BN + tid) * 4, rank + t);
     }
   };
 
   const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
   const int qa = ti.q0 + ra / G, qb = ti.q0 + rb / G;
-  const int ta = tauS[ra / G], tb = tauS[rb / G];
+  const int ta = DENSE ? 0 : tauS[ra / G], tb = DENSE ? 0 : tauS[rb / G];
   float o[P::NOT][4];
 #pragma unroll
   for (int n = 0; n < P::NOT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
@@ -432,8 +423,13 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
           const int e = j * P::BN + col;
           if (e >= nA) {
             const int t = posb[st * P::BN + col];
-            const int r = rkb[st * P::BN + col];
-            const bool kp = (c < 2) ? keep_key(qa, t, r, ta, a.s, a.w) : keep_key(qb, t, r, tb, a.s, a.w);
+            bool kp;
+            if (DENSE) {
+              kp = t <= ((c < 2) ? qa : qb);
+            } else {
+              const int r = rkb[st * P::BN + col];
+              kp = (c < 2) ? keep_key(qa, t, r, ta, a.s, a.w) : keep_key(qb, t, r, tb, a.s, a.w);
+            }
             if (e >= nU || !kp) v = -INFINITY;
           }
         }
@@ -468,6 +464,7 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
     }
     la = la * aa + sa;
     lb = lb * ab + sb;
+    if (WANT_Y) {
 #pragma unroll
     for (int n = 0; n < P::NOT; ++n) {
       o[n][0] *= aa;
@@ -491,6 +488,7 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
         mma_bf16(o[2 * np + 1], p0, p1, p2, p3, b2, b3);
       }
     }
+    }
     __syncthreads();
     if (j + 2 < nblk) issue(j + 2, st);
     cp_commit();
@@ -507,17 +505,21 @@ __global__ void __launch_bounds__(TcP<HD, G>::THREADS, 1) prompt_tc_kernel(Promp
   const size_t rowb = ((size_t)ti.seq * H * G + (size_t)ti.h * G + rb % G) * S + qb;
   const int col = 2 * (lane & 3);
   if (qa <= ti.q1) {
-    float* y = a.Y + rowa * HD + col;
+    if (WANT_Y) {
+      float* y = a.Y + rowa * HD + col;
 #pragma unroll
-    for (int n = 0; n < P::NOT; ++n)
-      *reinterpret_cast<float2*>(y + 8 * n) = make_float2(o[n][0] * ia, o[n][1] * ia);
+      for (int n = 0; n < P::NOT; ++n)
+        *reinterpret_cast<float2*>(y + 8 * n) = make_float2(o[n][0] * ia, o[n][1] * ia);
+    }
     if (a.lse && (lane & 3) == 0) a.lse[rowa] = (ma + __log2f(la)) * kLn2;
   }
   if (qb <= ti.q1) {
-    float* y = a.Y + rowb * HD + col;
+    if (WANT_Y) {
+      float* y = a.Y + rowb * HD + col;
 #pragma unroll
-    for (int n = 0; n < P::NOT; ++n)
-      *reinterpret_cast<float2*>(y + 8 * n) = make_float2(o[n][2] * ib, o[n][3] * ib);
+      for (int n = 0; n < P::NOT; ++n)
+        *reinterpret_cast<float2*>(y + 8 * n) = make_float2(o[n][2] * ib, o[n][3] * ib);
+    }
     if (a.lse && (lane & 3) == 0) a.lse[rowb] = (mb + __log2f(lb)) * kLn2;
   }
 }
@@ -538,24 +540,42 @@ size_t tc_smem(int capA, int capM) {
   return (size_t)TcP<HD, G>::OFF_LIST + (size_t)(capA + capM) * 4;
 }
 
-template <int HD, int G>
+template <int HD, int G, bool DENSE, bool WANT_Y>
 cudaError_t launch_tc(PromptArgs a, int n_pairs, cudaStream_t stream) {
   using P = TcP<HD, G>;
-  a.capM = a.s + 2 * P::BM + a.w;
+  if (DENSE) a.capA = a.capM = 0;
+  else a.capM = a.s + 2 * P::BM + a.w;
   const size_t smem = tc_smem<HD, G>(a.capA, a.capM);
   if (smem > 227 * 1024) return cudaErrorInvalidValue;
   dim3 grid((a.S + P::BM - 1) / P::BM, n_pairs);
-  return launch_cfg(prompt_tc_kernel<HD, G>, grid, P::THREADS, smem, stream, a);
+  return launch_cfg(prompt_tc_kernel<HD, G, DENSE, WANT_Y>, grid, P::THREADS, smem, stream, a);
 }
 
-template <typename T, int HD>
+template <typename T, int HD, bool DENSE>
 cudaError_t launch_simt(PromptArgs a, int n_pairs, cudaStream_t stream) {
-  a.capM = a.s + 2 * SIMT_BM + a.w;
+  if (DENSE) a.capA = a.capM = 0;
+  else a.capM = a.s + 2 * SIMT_BM + a.w;
   const size_t smem = (size_t)(SIMT_NT / 32) * HD * 4 + (SIMT_BM + SIMT_NT / 32 + 2) * 4 +
                       (size_t)(a.capA + a.capM) * 4;
   if (smem > 227 * 1024) return cudaErrorInvalidValue;
   dim3 grid((a.S + SIMT_BM - 1) / SIMT_BM, n_pairs);
-  return launch_cfg(prompt_simt_kernel<T, HD>, grid, SIMT_NT, smem, stream, a);
+  return launch_cfg(prompt_simt_kernel<T, HD, DENSE>, grid, SIMT_NT, smem, stream, a);
+}
+
+template <bool DENSE, bool WANT_Y>
+cudaError_t dispatch(const PromptArgs& a, int n_pairs, int dtype, int d, int G, cudaStream_t stream) {
+  if (dtype == KVPOP_BF16) {
+    if (d == 128) {
+      if (G == 4) return launch_tc<128, 4, DENSE, WANT_Y>(a, n_pairs, stream);
+      if (G == 2) return launch_tc<128, 2, DENSE, WANT_Y>(a, n_pairs, stream);
+      return launch_tc<128, 1, DENSE, WANT_Y>(a, n_pairs, stream);
+    }
+    if (G == 4) return launch_tc<64, 4, DENSE, WANT_Y>(a, n_pairs, stream);
+    if (G == 2) return launch_tc<64, 2, DENSE, WANT_Y>(a, n_pairs, stream);
+    return launch_tc<64, 1, DENSE, WANT_Y>(a, n_pairs, stream);
+  }
+  if (d == 128) return launch_simt<float, 128, DENSE>(a, n_pairs, stream);
+  return launch_simt<float, 64, DENSE>(a, n_pairs, stream);
 }
 
 }  // namespace
@@ -575,19 +595,15 @@ cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, co
   if (n_seq <= 0 || S <= 0) return cudaSuccess;
   PromptArgs a{Q, K, V, rank, tau, len, Y, lse, H, G, S, s, w, s + k, 0,
                1.4426950408889634f / sqrtf((float)d), err};
-  const int n_pairs = n_seq * H;
-  if (dtype == KVPOP_BF16) {
-    if (d == 128) {
-      if (G == 4) return launch_tc<128, 4>(a, n_pairs, stream);
-      if (G == 2) return launch_tc<128, 2>(a, n_pairs, stream);
-      return launch_tc<128, 1>(a, n_pairs, stream);
-    }
-    if (G == 4) return launch_tc<64, 4>(a, n_pairs, stream);
-    if (G == 2) return launch_tc<64, 2>(a, n_pairs, stream);
-    return launch_tc<64, 1>(a, n_pairs, stream);
-  }
-  if (d == 128) return launch_simt<float, 128>(a, n_pairs, stream);
-  return launch_simt<float, 64>(a, n_pairs, stream);
+  return dispatch<false, true>(a, n_seq * H, dtype, d, G, stream);
+}
+
+cudaError_t launch_causal_lse(const void* Q, const void* K, const int32_t* len, int n_seq, int H,
+                              int G, int d, int S, int dtype, float* lse, cudaStream_t stream) {
+  if (n_seq <= 0 || S <= 0) return cudaSuccess;
+  PromptArgs a{Q, K, nullptr, nullptr, nullptr, len, nullptr, lse, H, G, S, 0, 1, 0, 0,
+               1.4426950408889634f / sqrtf((float)d), nullptr};
+  return dispatch<true, false>(a, n_seq * H, dtype, d, G, stream);
 }
 
 }  // namespace kvpop

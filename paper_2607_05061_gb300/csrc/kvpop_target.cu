@@ -1,0 +1,349 @@
+// Future-attention target for training the scorer (Sec. 3.4, App. D, App. F.1-F.2).
+//
+// Kernel 1, the transposed attention pass (App. D.2): for every key t of KV
+// head h and every query head g of its group,
+//   log mbar_t^(g) = LSE over d in [t + w, S - 1] (and d <= t + w + L with a
+//                    lookahead L) of  q_d^(g) . k_t / sqrt(d_k) - LSE_d^(g),
+// where LSE_d is the dense causal normaliser (exact target) or the sparse one
+// returned by the prompt attention (App. D.3).  Keys play the queries: a CTA
+// holds 128 keys of one (sequence, KV head) as the A operand in registers and
+// streams the query rows of each head g past them in blocks of 64 (B operand,
+// 16-byte cp.async into a swizzled double buffer) with the per-column LSE_d in
+// shared memory; only a running max and sum are kept per (key, head) -- the
+// value output of the pass is never formed.  bf16 on m16n8k16 tensor-core
+// MMAs, fp32 on CUDA cores (one warp per (key, head), 32 queries per round).
+//
+// Kernel 2 aggregates per KV head (Eq. 2, App. F.1-F.2):
+//   r_t = log(eps + Agg_g mbar_t^(g) / N_t),  N_t = max(1, S - (t + w)),
+// N_t clipped to L + 1 with a lookahead, Agg = max or mean; without count
+// normalisation N_t = 1.
+#include "kvpop_mma.cuh"
+
+namespace kvpop {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2f = 0.69314718055994530942f;
+
+struct TargetArgs {
+  const void* Q;             // [n][H*G][S][d]
+  const void* K;             // [n][H][S][d]
+  const float* lse;          // [n][H*G][S] natural log
+  const int32_t* len;        // [n] or nullptr
+  float* logm;               // [n][H*G][S] out
+  int H, G, S, w, la;
+  float kscale;              // log2(e) / sqrt(d)
+};
+
+__device__ __forceinline__ int row_len(const TargetArgs& a, int seq) {
+  return a.len ? max(0, min(a.len[seq], a.S)) : a.S;
+}
+
+// last query position that may attend to key t (-1 if none)
+__device__ __forceinline__ int future_hi(int t, int L, int w, int la) {
+  const int hi = la > 0 ? min(L - 1, t + w + la) : L - 1;
+  return t + w <= hi ? hi : -1;
+}
+
+// ---------------------------------------------------------------- CUDA-core kernel
+constexpr int TS_NT = 256;
+constexpr int TS_BT = 32;
+
+template <typename T, int HD>
+__global__ void __launch_bounds__(TS_NT) target_simt_kernel(TargetArgs a) {
+  __shared__ float kv[TS_NT / 32][HD];
+  constexpr int NW = TS_NT / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int pair = blockIdx.y, seq = pair / a.H, h = pair - seq * a.H;
+  const int G = a.G, S = a.S, L = row_len(a, seq);
+  const int t0 = blockIdx.x * TS_BT;
+  if (t0 >= L) return;
+  const T* Kp = static_cast<const T*>(a.K) + (size_t)pair * S * HD;
+  float* k_s = kv[warp];
+  for (int r = warp; r < TS_BT * G; r += NW) {
+    const int tl = r / G, g = r - tl * G, t = t0 + tl;
+    if (t >= L) break;
+    const size_t qrow = (size_t)seq * a.H * G + (size_t)h * G + g;
+    const T* Qg = static_cast<const T*>(a.Q) + qrow * S * HD;
+    const float* lse = a.lse + qrow * S;
+    for (int i = lane; i < HD; i += 32) k_s[i] = to_f(Kp[(size_t)t * HD + i]) * a.kscale;
+    __syncwarp();
+    const int hi = future_hi(t, L, a.w, a.la);
+    float m = -INFINITY, l = 0.f;
+    if (hi >= 0) {
+      for (int d0 = t + a.w; d0 <= hi; d0 += 32) {
+        const int d = d0 + lane;
+        float v = -INFINITY;
+        if (d <= hi) {
+          const T* qr = Qg + (size_t)d * HD;
+          float acc = 0.f;
+#pragma unroll 8
+          for (int i = 0; i < HD; ++i) acc = fmaf(k_s[i], to_f(qr[i]), acc);
+          v = acc - lse[d] * kLog2e;
+        }
+        float mx = v;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float mn = fmaxf(m, mx);
+        const float u = mn == -INFINITY ? 0.f : mn;
+        float p = d <= hi ? exp2f(v - u) : 0.f;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
+        l = l * exp2f(m - u) + p;
+        m = mn;
+      }
+    }
+    if (lane == 0) a.logm[qrow * S + t] = l > 0.f ? (m + log2f(l)) * kLn2f : -INFINITY;
+    __syncwarp();
+  }
+}
+
+// ---------------------------------------------------------------- tensor-core kernel
+template <int HD>
+struct TgP {
+  static constexpr int NW = 8;
+  static constexpr int THREADS = NW * 32;
+  static constexpr int ROWS = 16 * NW;             // keys per CTA
+  static constexpr int BN = 64;                    // queries per block
+  static constexpr int NKS = HD / 16;
+  static constexpr int NNT = BN / 8;
+  static constexpr int CH = HD / 8;
+  static constexpr int ROWB = HD * 2;
+  static constexpr int QB = BN * ROWB;
+  static constexpr int STAGES = 2;
+  static constexpr int OFF_LSE = STAGES * QB;
+  static constexpr int SMEM = OFF_LSE + STAGES * BN * 4;
+  static_assert(ROWS * ROWB <= STAGES * QB, "the key tile is staged in the query buffers");
+};
+
+template <int HD>
+__global__ void __launch_bounds__(TgP<HD>::THREADS, 1) target_tc_kernel(TargetArgs a) {
+  using P = TgP<HD>;
+  extern __shared__ __align__(1024) unsigned char smem_tg[];
+  float* lseS = reinterpret_cast<float*>(smem_tg + P::OFF_LSE);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int pair = blockIdx.y, seq = pair / a.H, h = pair - seq * a.H;
+  const int G = a.G, S = a.S, L = row_len(a, seq), w = a.w, la = a.la;
+  const int t0 = blockIdx.x * P::ROWS;
+  if (t0 >= L) return;
+  const int t1 = min(t0 + P::ROWS - 1, L - 1);
+  const size_t qrow0 = (size_t)seq * a.H * G + (size_t)h * G;
+  const int d_lo = t0 + w;
+  const int d_hi = la > 0 ? min(L - 1, t1 + w + la) : L - 1;
+  const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
+  const int ta = t0 + ra, tb = t0 + rb;
+  if (d_lo > d_hi) {                               // no key of the tile has a future query
+    for (int i = tid; i < (t1 - t0 + 1) * G; i += P::THREADS) {
+      const int tl = i / G, g = i - tl * G;
+      a.logm[(qrow0 + g) * S + t0 + tl] = -INFINITY;
+    }
+    return;
+  }
+  const int nblk = (d_hi - d_lo + P::BN) / P::BN;
+  const int total = G * nblk;
+  const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(smem_tg);
+  const bf16* Kp = static_cast<const bf16*>(a.K) + (size_t)pair * S * HD;
+
+  // key tile -> query buffers (rows past the sequence zero-filled) -> A fragments
+  for (int i = tid; i < P::ROWS * P::CH; i += P::THREADS) {
+    const int r = i / P::CH, c = i - r * P::CH;
+    const bool ok = t0 + r <= t1;
+    cp_async16(sbase + swz(r, c, P::ROWB), Kp + (size_t)(ok ? t0 + r : t0) * HD + c * 8, ok ? 16 : 0);
+  }
+  cp_commit();
+  cp_wait<0>();
+  __syncthreads();
+  uint32_t kf[P::NKS][4];
+#pragma unroll
+  for (int ks = 0; ks < P::NKS; ++ks) {
+    const int r = 16 * warp + ((lane >> 3) & 1) * 8 + (lane & 7);
+    const int c = 2 * ks + (lane >> 4);
+    ldsm_x4(sbase + swz(r, c, P::ROWB), kf[ks][0], kf[ks][1], kf[ks][2], kf[ks][3]);
+  }
+  __syncthreads();
+
+  auto issue = [&](int j, int st) {
+    const int g = j / nblk, b = j - g * nblk;
+    const int d0 = d_lo + b * P::BN;
+    const bf16* Qg = static_cast<const bf16*>(a.Q) + (qrow0 + g) * S * HD;
+    const uint32_t dst = sbase + st * P::QB;
+    for (int i = tid; i < P::BN * P::CH; i += P::THREADS) {
+      const int r = i / P::CH, c = i - r * P::CH;
+      const bool ok = d0 + r <= d_hi;
+      cp_async16(dst + swz(r, c, P::ROWB), Qg + (size_t)(ok ? d0 + r : d0) * HD + c * 8, ok ? 16 : 0);
+    }
+    if (tid < P::BN) {
+      const float* lse = a.lse + (qrow0 + g) * S;
+      if (d0 + tid <= d_hi)
+        cp_async4(sbase + P::OFF_LSE + (st * P::BN + tid) * 4, lse + d0 + tid);
+      else
+        lseS[st * P::BN + tid] = 0.f;
+    }
+  };
+
+  const int hia = future_hi(ta, L, w, la), hib = future_hi(tb, L, w, la);
+  float ma = -INFINITY, mb = -INFINITY, la_ = 0.f, lb_ = 0.f;
+  issue(0, 0);
+  cp_commit();
+  if (total > 1) issue(1, 1);
+  cp_commit();
+  for (int j = 0; j < total; ++j) {
+    const int st = j & 1;
+    const int g = j / nblk, b = j - g * nblk;
+    const int d0 = d_lo + b * P::BN;
+    cp_wait<1>();
+    __syncthreads();
+    const uint32_t qb = sbase + st * P::QB;
+    float sc[P::NNT][4];
+#pragma unroll
+    for (int n = 0; n < P::NNT; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < P::NKS; ++ks) {
+#pragma unroll
+      for (int np = 0; np < P::NNT / 2; ++np) {
+        const int r = 8 * (2 * np + (lane >> 4)) + (lane & 7);
+        const int c = 2 * ks + ((lane >> 3) & 1);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(qb + swz(r, c, P::ROWB), b0, b1, b2, b3);
+        mma_bf16(sc[2 * np], kf[ks][0], kf[ks][1], kf[ks][2], kf[ks][3], b0, b1);
+        mma_bf16(sc[2 * np + 1], kf[ks][0], kf[ks][1], kf[ks][2], kf[ks][3], b2, b3);
+      }
+    }
+    // rows need a mask where the block reaches below t + w, past t + w + L, or past the end
+    const bool masked = d0 < t1 + w || d0 + P::BN - 1 > d_hi || (la > 0 && d0 + P::BN - 1 > t0 + w + la);
+    float mxa = -INFINITY, mxb = -INFINITY;
+#pragma unroll
+    for (int n = 0; n < P::NNT; ++n) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int col = n * 8 + 2 * (lane & 3) + (c & 1);
+        const int d = d0 + col;
+        float v = sc[n][c] * a.kscale - lseS[st * P::BN + col] * kLog2e;
+        if (masked) {
+          const int t = c < 2 ? ta : tb;
+          const int hi = c < 2 ? hia : hib;
+          if (d < t + w || d > hi) v = -INFINITY;
+        }
+        sc[n][c] = v;
+      }
+      mxa = fmaxf(mxa, fmaxf(sc[n][0], sc[n][1]));
+      mxb = fmaxf(mxb, fmaxf(sc[n][2], sc[n][3]));
+    }
+#pragma unroll
+    for (int o = 1; o <= 2; o <<= 1) {
+      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, o));
+      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, o));
+    }
+    const float mna = fmaxf(ma, mxa), mnb = fmaxf(mb, mxb);
+    const float ua = mna == -INFINITY ? 0.f : mna, ub = mnb == -INFINITY ? 0.f : mnb;
+    float sa = 0.f, sb = 0.f;
+#pragma unroll
+    for (int n = 0; n < P::NNT; ++n) {
+      sa += ex2(sc[n][0] - ua) + ex2(sc[n][1] - ua);
+      sb += ex2(sc[n][2] - ub) + ex2(sc[n][3] - ub);
+    }
+    la_ = la_ * ex2(ma - ua) + sa;
+    lb_ = lb_ * ex2(mb - ub) + sb;
+    ma = mna;
+    mb = mnb;
+    if (b == nblk - 1) {                           // head g done: write and reset
+      float sa2 = la_, sb2 = lb_;
+#pragma unroll
+      for (int o = 1; o <= 2; o <<= 1) {
+        sa2 += __shfl_xor_sync(0xffffffffu, sa2, o);
+        sb2 += __shfl_xor_sync(0xffffffffu, sb2, o);
+      }
+      if ((lane & 3) == 0) {
+        float* out = a.logm + (qrow0 + g) * S;
+        if (ta <= t1) out[ta] = sa2 > 0.f ? (ma + __log2f(sa2)) * kLn2f : -INFINITY;
+        if (tb <= t1) out[tb] = sb2 > 0.f ? (mb + __log2f(sb2)) * kLn2f : -INFINITY;
+      }
+      ma = mb = -INFINITY;
+      la_ = lb_ = 0.f;
+    }
+    __syncthreads();
+    if (j + 2 < total) issue(j + 2, st);
+    cp_commit();
+  }
+  cp_wait<0>();
+}
+
+// ---------------------------------------------------------------- aggregation
+struct AggArgs {
+  const float* logm;         // [n][H*G][S]
+  const int32_t* len;
+  float* target;             // [n][H][S]
+  int n_pairs, H, G, S, w, la, agg, count_norm;
+  float log_eps;             // log(eps), -inf for eps = 0
+};
+
+__global__ void aggregate_kernel(AggArgs a) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)a.n_pairs * a.S) return;
+  const int pair = (int)(i / a.S), t = (int)(i - (size_t)pair * a.S);
+  const int seq = pair / a.H, h = pair - seq * a.H;
+  const int L = a.len ? max(0, min(a.len[seq], a.S)) : a.S;
+  if (t >= L) return;
+  float logN = 0.f;
+  if (a.count_norm) {
+    int n = max(1, L - (t + a.w));
+    if (a.la > 0) n = min(n, a.la + 1);
+    logN = logf((float)n);
+  }
+  const float* lm = a.logm + ((size_t)seq * a.H * a.G + (size_t)h * a.G) * a.S + t;
+  float x;
+  if (a.agg == 0) {
+    x = -INFINITY;
+    for (int g = 0; g < a.G; ++g) x = fmaxf(x, lm[(size_t)g * a.S]);
+  } else {
+    float mx = -INFINITY;
+    for (int g = 0; g < a.G; ++g) mx = fmaxf(mx, lm[(size_t)g * a.S]);
+    float sum = 0.f;
+    if (mx != -INFINITY)
+      for (int g = 0; g < a.G; ++g) sum += expf(lm[(size_t)g * a.S] - mx);
+    x = mx == -INFINITY ? -INFINITY : mx + logf(sum / (float)a.G);
+  }
+  x -= logN;
+  // log(eps + exp(x)) without overflow
+  const float hi = fmaxf(a.log_eps, x), lo = fminf(a.log_eps, x);
+  a.target[i] = lo == -INFINITY ? hi : hi + log1pf(expf(lo - hi));
+}
+
+}  // namespace
+
+cudaError_t launch_future_target(const void* Q, const void* K, const float* lse, const int32_t* len,
+                                 int n_seq, int H, int G, int d, int S, int w, int la, int dtype,
+                                 float* logm, float* target, int agg, int count_norm, float eps,
+                                 cudaStream_t stream) {
+  if (n_seq <= 0 || S <= 0) return cudaSuccess;
+  TargetArgs a{Q, K, lse, len, logm, H, G, S, w, la, 1.4426950408889634f / sqrtf((float)d)};
+  const int n_pairs = n_seq * H;
+  if (dtype == KVPOP_BF16) {
+    const size_t smem = d == 128 ? TgP<128>::SMEM : TgP<64>::SMEM;
+    dim3 grid((S + TgP<128>::ROWS - 1) / TgP<128>::ROWS, n_pairs);
+    if (d == 128) {
+      cudaError_t e = cudaFuncSetAttribute(target_tc_kernel<128>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      target_tc_kernel<128><<<grid, TgP<128>::THREADS, smem, stream>>>(a);
+    } else {
+      cudaError_t e = cudaFuncSetAttribute(target_tc_kernel<64>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      target_tc_kernel<64><<<grid, TgP<64>::THREADS, smem, stream>>>(a);
+    }
+  } else {
+    dim3 grid((S + TS_BT - 1) / TS_BT, n_pairs);
+    if (d == 128) target_simt_kernel<float, 128><<<grid, TS_NT, 0, stream>>>(a);
+    else target_simt_kernel<float, 64><<<grid, TS_NT, 0, stream>>>(a);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !target) return e;
+  AggArgs g{logm, len, target, n_pairs, H, G, S, w, la, agg, count_norm,
+            eps > 0.f ? logf(eps) : -INFINITY};
+  const size_t n = (size_t)n_pairs * S;
+  aggregate_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(g);
+  return cudaGetLastError();
+}
+
+}  // namespace kvpop

@@ -73,6 +73,11 @@ _SIGS = {
     "kvpop_prompt_attention": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, c_int32, c_int32, c_int32,
                                               c_int32, c_int32, c_int32, c_int32, c_int32,
                                               ctypes.c_int, _P, _P, _P]),
+    "kvpop_causal_lse": (ctypes.c_int, [_P, _P, _P, c_int32, c_int32, c_int32, c_int32, c_int32,
+                                        ctypes.c_int, _P, _P]),
+    "kvpop_future_target": (ctypes.c_int, [_P, _P, _P, _P, c_int32, c_int32, c_int32, c_int32, c_int32,
+                                           c_int32, c_int32, ctypes.c_int, _P, _P, c_int32, c_int32,
+                                           c_float, _P]),
     "kvpop_last_error": (ctypes.c_char_p, []),
     "kvpop_debug_fail_alloc_after": (None, [c_int32]),
 }
@@ -249,6 +254,35 @@ def prompt_attention(Q, K, V, rank, tau, n_sink: int, window: int, k: int, lengt
                                H, G, d, S, n_sink, window, k, dtype_code(K.dtype), _ptr(Y), _ptr(lse),
                                _stream(stream)), "kvpop_prompt_attention")
     return Y, lse
+
+
+def causal_lse(Q, K, lengths=None, lse=None, stream=None):
+    """Dense causal log-normalisers ``[n][H*G][S]`` (fp32) of ``Q [n][H*G][S][d]`` against
+    ``K [n][H][S][d]``."""
+    n_seq, H, S, d = K.shape
+    G = Q.shape[1] // H
+    lse = torch.empty((n_seq, H * G, S), dtype=torch.float32, device=K.device) if lse is None else lse
+    _ck(kvpop_causal_lse(_ptr(Q), _ptr(K), _ptr(lengths), n_seq, H, G, d, S, dtype_code(K.dtype),
+                         _ptr(lse), _stream(stream)), "kvpop_causal_lse")
+    return lse
+
+
+def future_target(Q, K, lse, window: int, lookahead: int = 0, agg: str = "max",
+                  count_norm: bool = True, eps: float = 1e-6, lengths=None, want_target: bool = True,
+                  logm=None, target=None, stream=None):
+    """Per-head future log masses ``[n][H*G][S]`` and, optionally, the per-KV-head target
+    ``[n][H][S]`` (both fp32)."""
+    n_seq, H, S, d = K.shape
+    G = Q.shape[1] // H
+    dev = K.device
+    logm = torch.empty((n_seq, H * G, S), dtype=torch.float32, device=dev) if logm is None else logm
+    if target is None and want_target:
+        target = torch.empty((n_seq, H, S), dtype=torch.float32, device=dev)
+    _ck(kvpop_future_target(_ptr(Q), _ptr(K), _ptr(lse), _ptr(lengths), n_seq, H, G, d, S, window,
+                            lookahead, dtype_code(K.dtype), _ptr(logm), _ptr(target),
+                            0 if agg == "max" else 1, int(bool(count_norm)), float(eps),
+                            _stream(stream)), "kvpop_future_target")
+    return logm, target
 
 
 def parse_state(blob: bytes, cfg: kvpop_config) -> dict:

@@ -117,3 +117,31 @@ def test_topk_and_prompt_attention_reject_bad_arguments(kv):
     assert att(*args(Q=P + 8)) == align
     assert att(*args(Y=P + 4)) == align
     assert att(*args(lse=P + 2)) == align
+
+
+def test_causal_lse_and_future_target_reject_bad_arguments(kv):
+    P = 0x1000
+    bad, align = 1, 2
+    lse = kv.kvpop_causal_lse
+    assert lse(P, P, None, 0, 8, 4, 128, 64, 1, P, None) == 0
+    assert lse(P, P, None, 2, 8, 4, 96, 64, 1, P, None) == bad          # head_dim
+    assert lse(P, P, None, 2, 8, 4, 128, 64, 5, P, None) == bad         # dtype
+    assert lse(P, P, None, 2, 8, 4, 128, 64, 1, None, None) == bad
+    assert lse(P + 8, P, None, 2, 8, 4, 128, 64, 1, P, None) == align
+    ft = kv.kvpop_future_target
+    args = lambda **o: [o.get(n, v) for n, v in (
+        ("Q", P), ("K", P), ("lse", P), ("len", None), ("n", 2), ("H", 8), ("G", 4), ("d", 128),
+        ("S", 64), ("w", 16), ("la", 0), ("dt", 1), ("logm", P), ("tgt", P), ("agg", 0), ("cn", 1),
+        ("eps", 1e-6), ("st", None))]
+    assert ft(*args(n=0)) == 0
+    assert ft(*args(w=-1)) == bad
+    assert ft(*args(la=-3)) == bad
+    assert ft(*args(agg=2)) == bad
+    assert ft(*args(cn=3)) == bad
+    assert ft(*args(eps=-1.0)) == bad
+    assert ft(*args(eps=float("nan"))) == bad
+    assert ft(*args(eps=float("inf"))) == bad
+    assert ft(*args(logm=None)) == bad
+    assert ft(*args(G=3)) == bad
+    assert ft(*args(lse=P + 2)) == align
+    assert ft(*args(tgt=P + 1)) == align
