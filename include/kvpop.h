@@ -68,16 +68,23 @@ typedef struct {
   kvpop_dtype kv_dtype;   /* element type of q, k, v and the K/V store         */
 } kvpop_config;
 
-/* Scorer parameters (Sec. 3.3 / App. E.2 two-layer MLP, GELU(erf) hidden layer).
- * Host or device fp32 arrays; copied into the cache at init (caller keeps
- * ownership).  Input order of W1's rows: [k (d); v (d); qbar (d)]. */
+/* Stateless scorer parameters (Sec. 3.3, App. E.2): the per-head two-layer MLP
+ *   r = w2 . act(W1^T x + b1) + b2
+ * on x = [k (d); v (d); qbar (d)] (input_kind 0; qbar = mean of the next D
+ * queries over the G heads) or x = [k; v] (input_kind 1, the plain SiLU-MLP
+ * scorer of Sec. 3.3), with act = GELU(erf) (activation 0), SiLU (1) or the
+ * identity (2, a linear scorer when F = 1 and w2 = 1).  Host or device fp32
+ * arrays; copied into the cache at init (caller keeps ownership).  A zeroed
+ * struct with the five pointers set is the GELU [k; v; qbar] scorer. */
 typedef struct {
-  const float* W1;         /* [H][3d][F]                                      */
+  const float* W1;         /* [H][3d][F], or [H][2d][F] with input_kind 1     */
   const float* b1;         /* [H][F]                                          */
   const float* w2;         /* [H][F]                                          */
   const float* b2;         /* [H]                                             */
   const float* log_gamma;  /* [H] per-head log decay (App. B.3, n = 1) or NULL
                               for none; stored priority = r - u * log_gamma   */
+  int32_t input_kind;      /* 0: [k; v; qbar]   1: [k; v]                     */
+  int32_t activation;      /* 0: GELU (erf)   1: SiLU   2: identity           */
 } kvpop_scorer;
 
 /* Stateful delayed mLSTM scorer (App. A, App. E.3, App. E.4), per KV head.

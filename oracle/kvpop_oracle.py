@@ -12,7 +12,9 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
   context gathered meanwhile (Sec. 3.3 "Stateful scorers"; App. E.4).  The
   scorer is the stateless two-layer MLP of Sec. 3.3 / App. E.2 applied to the
   input [k_u; v_u; qbar_u], where qbar_u averages the D queries u+1..u+D over
-  the G query heads that share the KV head, with an exact-erf GELU hidden layer.
+  the G query heads that share the KV head, with an exact-erf GELU hidden layer;
+  or the paper's plain variant on [k_u; v_u] (W1 with 2d rows), with a SiLU or
+  identity hidden layer.
 * Static priority for decay step n = 1: rbar = r - u * log(gamma_h)
   (App. B.3); with log(gamma) = 0 it is the raw score.
 * Running top-k under a fixed budget (Sec. 3.2 "Running top-k sparse
@@ -42,7 +44,7 @@ from dataclasses import dataclass
 from typing import Optional
 
 import numpy as np
-from scipy.special import erf
+from scipy.special import erf, expit
 
 _SQRT1_2 = 1.0 / np.sqrt(2.0)
 
@@ -58,12 +60,14 @@ class OracleParams:
     delay_D: int
     n_sink: int = 0
     log_gamma: float = 0.0
+    activation: str = "gelu"   # gelu / silu / identity
 
     @staticmethod
-    def for_head(W1, b1, w2, b2, log_gamma, h, budget_B, delay_D, n_sink=0):
+    def for_head(W1, b1, w2, b2, log_gamma, h, budget_B, delay_D, n_sink=0, activation="gelu"):
         as64 = lambda a: np.asarray(a, dtype=np.float64)
         return OracleParams(as64(W1[h]), as64(b1[h]), as64(w2[h]), float(as64(b2[h])),
-                            int(budget_B), int(delay_D), int(n_sink), float(np.float32(log_gamma[h])))
+                            int(budget_B), int(delay_D), int(n_sink), float(np.float32(log_gamma[h])),
+                            activation)
 
 
 def gelu_erf(z):
@@ -71,13 +75,19 @@ def gelu_erf(z):
     return 0.5 * z * (1.0 + erf(z * _SQRT1_2))
 
 
-def scorer_mlp(x: np.ndarray, p: OracleParams) -> np.ndarray:
-    """Two-layer headwise MLP score (Sec. 3.3, App. E.2): w2 . GELU(W1^T x + b1) + b2.
+def silu(z):
+    """SiLU(z) = z * sigmoid(z)."""
+    return z * expit(z)
 
-    ``x`` is ``[3d]`` or ``[n][3d]``; returns fp64 scores.
+
+def scorer_mlp(x: np.ndarray, p: OracleParams) -> np.ndarray:
+    """Two-layer headwise MLP score (Sec. 3.3, App. E.2): w2 . act(W1^T x + b1) + b2.
+
+    ``x`` is ``[I]`` or ``[n][I]`` (I = rows of W1); returns fp64 scores.
     """
     z = x @ p.W1 + p.b1
-    return gelu_erf(z) @ p.w2 + p.b2
+    act = {"gelu": gelu_erf, "silu": silu, "identity": lambda y: y}[p.activation]
+    return act(z) @ p.w2 + p.b2
 
 
 def round_score(r64) -> np.float32:
@@ -123,6 +133,8 @@ class HeadCache:
         later = [e[3] for e in list(self.pending)[1:]]          # qmean(u+1 .. p-1)
         qbar = (np.sum(later, axis=0) if later else 0.0) + qmean_p
         qbar = qbar / self.p.delay_D
+        if self.p.W1.shape[0] == 2 * self.d:          # the [k; v] scorer
+            return u, np.concatenate([k_u, v_u])
         return u, np.concatenate([k_u, v_u, qbar])
 
     # ---- Sec. 3.2 / App. C.1 keep-or-drop under the budget ---------------------------
@@ -222,6 +234,8 @@ def prefill_head(p: OracleParams, Q: np.ndarray, K: np.ndarray, V: np.ndarray,
                 qsum += qmean[j:j + n_elig]
             qbar = qsum / D
             X = np.concatenate([K[:n_elig], V[:n_elig], qbar], axis=1)
+            if p.W1.shape[0] == 2 * head_dim:
+                X = X[:, : 2 * head_dim]
             r64 = scorer_mlp(X, p)
         else:
             r64 = np.asarray(override[:n_elig], dtype=np.float64)

@@ -33,7 +33,7 @@ class PairTrace:
 def head_params(cfg, weights, h: int) -> OracleParams:
     W1, b1, w2, b2, lg = weights
     return OracleParams.for_head(W1.numpy(), b1.numpy(), w2.numpy(), b2.numpy(), lg.numpy(),
-                                 h, cfg.budget_B, cfg.delay_D, cfg.n_sink)
+                                 h, cfg.budget_B, cfg.delay_D, cfg.n_sink, cfg.scorer_act)
 
 
 def prefill_pair(cfg, weights, b: int, h: int, prompt_len: int,

@@ -190,6 +190,8 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
   kvpop_status vs = validate(cfg);
   if (vs != KVPOP_OK) return vs;
   if (sc && (!sc->W1 || !sc->b1 || !sc->w2 || !sc->b2)) return KVPOP_ERR_INVALID_ARG;
+  if (sc && (sc->input_kind < 0 || sc->input_kind > 1 || sc->activation < 0 || sc->activation > 2))
+    return KVPOP_ERR_INVALID_ARG;
   if (ms && (!ms->Wq || !ms->Wk || !ms->Wv || !ms->wi || !ms->wf || !ms->bi || !ms->bf || !ms->a ||
              !ms->b))
     return KVPOP_ERR_INVALID_ARG;
@@ -202,6 +204,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
   dm.batch = cfg->batch; dm.H = cfg->n_kv_heads; dm.G = cfg->q_per_kv; dm.d = cfg->head_dim;
   dm.B = cfg->budget_B; dm.D = cfg->delay_D; dm.s = cfg->n_sink; dm.F = cfg->scorer_hidden;
   dm.Fp = (dm.F + 3) & ~3;
+  dm.act = sc ? sc->activation : 0;
   dm.dtype = cfg->kv_dtype;
   dm.pairs = dm.batch * dm.H;
   c->esz = cfg->kv_dtype == KVPOP_F32 ? 4 : 2;
@@ -212,7 +215,8 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
 
   const size_t pairs = dm.pairs, B = dm.B, D = dm.D, d = dm.d, H = dm.H, F = dm.F, Fp = dm.Fp;
   const size_t NB = min_blocks(dm.B);
-  const size_t I = 3 * d;
+  const size_t I = 3 * d;                              // device rows of W1: [k; v; qbar]
+  const size_t Isrc = (sc && sc->input_kind == 1) ? 2 * d : I;   // rows the caller gives
   AttendConfig ac;
   c->use_tc = cfg->kv_dtype == KVPOP_BF16;
   kvpop_status s = from_cuda(NOTE(c->use_tc ? tc_config(dm, &ac) : attend_config(dm, &ac)));
@@ -295,8 +299,10 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     c->st.W1 = W1; c->st.b1 = b1; c->st.w2 = w2; c->st.b2 = b2;
     // hidden units padded to Fp with zero weights: rows of F floats into rows of Fp
     cudaError_t e = NOTE(cudaMemsetAsync(w, 0, wbytes, stream));
-    if (e == cudaSuccess && sc)
-      e = NOTE(cudaMemcpy2DAsync(W1, Fp * 4, sc->W1, F * 4, F * 4, H * I, cudaMemcpyDefault, stream));
+    // a [k; v]-only scorer keeps zero weights on the qbar rows
+    for (size_t h = 0; h < H && e == cudaSuccess && sc; ++h)
+      e = NOTE(cudaMemcpy2DAsync(W1 + h * I * Fp, Fp * 4, sc->W1 + h * Isrc * F, F * 4, F * 4, Isrc,
+                                 cudaMemcpyDefault, stream));
     if (e == cudaSuccess && sc)
       e = NOTE(cudaMemcpy2DAsync(b1, Fp * 4, sc->b1, F * 4, F * 4, H, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && sc)
@@ -341,8 +347,8 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
           if (f0 >= F) break;
           const size_t wcols = (F - f0 < FS) ? F - f0 : FS;
           const size_t sl = h * 8 + r;
-          e = NOTE(cudaMemcpy2DAsync(c->W1s + sl * I * FS, FS * 4, sc->W1 + h * I * F + f0, F * 4,
-                                     wcols * 4, I, cudaMemcpyDefault, stream));
+          e = NOTE(cudaMemcpy2DAsync(c->W1s + sl * I * FS, FS * 4, sc->W1 + h * Isrc * F + f0, F * 4,
+                                     wcols * 4, Isrc, cudaMemcpyDefault, stream));
           if (e == cudaSuccess)
             e = NOTE(cudaMemcpyAsync(c->b1s + sl * FS, sc->b1 + h * F + f0, wcols * 4,
                                      cudaMemcpyDefault, stream));

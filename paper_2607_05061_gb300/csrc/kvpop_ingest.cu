@@ -203,7 +203,7 @@ __global__ void __launch_bounds__(NT) ingest_kernel(IngestArgs<T> a) {
     if (f < Fp) {
       const float wf = f < F ? w2[f] : 0.f;
 #pragma unroll
-      for (int r = 0; r < SB; ++r) contrib[r * Fp + f] = wf * gelu_erf(acc[u][r]);
+      for (int r = 0; r < SB; ++r) contrib[r * Fp + f] = wf * scorer_act(acc[u][r], a.dm.act);
     }
   }
   if (tid == 0 && !ok) {

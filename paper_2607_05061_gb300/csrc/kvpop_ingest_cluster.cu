@@ -282,8 +282,8 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
         a1 = fmaf(u1.x, w0, a1); a1 = fmaf(u1.y, w1, a1); a1 = fmaf(u1.z, w2, a1); a1 = fmaf(u1.w, w3, a1);
       }
       const float wf = w2s[f];
-      c0 = fmaf(wf, gelu_erf(a0), c0);
-      c1 = fmaf(wf, gelu_erf(a1), c1);
+      c0 = fmaf(wf, scorer_act(a0, dm.act), c0);
+      c1 = fmaf(wf, scorer_act(a1, dm.act), c1);
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {

@@ -52,6 +52,7 @@ struct State {                 // device pointers of one cache
 
 struct Dims {
   int batch, H, G, d, B, D, s, F, Fp;
+  int act;                     // scorer hidden activation: 0 GELU (erf), 1 SiLU, 2 identity
   int dtype;                   // kvpop_dtype
   int pairs;
 };
@@ -167,6 +168,13 @@ __device__ __forceinline__ float static_priority(float r, int u, const float* lo
 // Exact-erf GELU.
 __device__ __forceinline__ float gelu_erf(float z) {
   return 0.5f * z * (1.0f + erff(z * 0.70710678118654752440f));
+}
+
+// Hidden-layer activation of the stateless scorer (Sec. 3.3): GELU, SiLU or none.
+__device__ __forceinline__ float scorer_act(float z, int act) {
+  if (act == 0) return gelu_erf(z);
+  if (act == 1) return z / (1.0f + expf(-z));
+  return z;
 }
 
 }  // namespace kvpop

@@ -145,7 +145,7 @@ __global__ void __launch_bounds__(NT1) prefill_score_kernel(ScoreArgs<T> a) {
     }
     const float wf = w2[f];
 #pragma unroll
-    for (int r = 0; r < UT; ++r) part[r] = fmaf(wf, gelu_erf(acc[r]), part[r]);
+    for (int r = 0; r < UT; ++r) part[r] = fmaf(wf, scorer_act(acc[r], dm.act), part[r]);
   }
 #pragma unroll
   for (int r = 0; r < UT; ++r) red[r * NT1 + threadIdx.x] = part[r];

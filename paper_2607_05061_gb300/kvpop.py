@@ -36,7 +36,10 @@ class kvpop_config(ctypes.Structure):
 
 class kvpop_scorer(ctypes.Structure):
     _fields_ = [("W1", c_void_p), ("b1", c_void_p), ("w2", c_void_p), ("b2", c_void_p),
-                ("log_gamma", c_void_p)]
+                ("log_gamma", c_void_p), ("input_kind", c_int32), ("activation", c_int32)]
+
+
+ACTIVATIONS = {"gelu": 0, "silu": 1, "identity": 2}
 
 
 class kvpop_mlstm_scorer(ctypes.Structure):
@@ -126,9 +129,12 @@ class KVpopCache:
 
     def __init__(self, batch: int, n_kv_heads: int, q_per_kv: int, head_dim: int, budget_B: int,
                  delay_D: int, scorer_hidden: int, kv_dtype, W1=None, b1=None, w2=None, b2=None,
-                 log_gamma=None, n_sink: int = 0, stream=None, mlstm: Optional[dict] = None):
-        """MLP scorer from ``W1, b1, w2, b2``; or, with ``mlstm`` (a dict of ``Wq, Wk, Wv,
-        wi, wf, bi, bf, a, b`` and optionally ``log_gamma``), the stateful mLSTM scorer."""
+                 log_gamma=None, n_sink: int = 0, stream=None, mlstm: Optional[dict] = None,
+                 activation: str = "gelu", kv_only: bool = False):
+        """MLP scorer from ``W1, b1, w2, b2`` (``W1 [H][3d][F]`` on [k; v; qbar], or
+        ``[H][2d][F]`` on [k; v] with ``kv_only``; hidden ``activation`` gelu / silu /
+        identity); or, with ``mlstm`` (a dict of ``Wq, Wk, Wv, wi, wf, bi, bf, a, b`` and
+        optionally ``log_gamma``), the stateful mLSTM scorer."""
         self.cfg = kvpop_config(batch, n_kv_heads, q_per_kv, head_dim, budget_B, delay_D, n_sink,
                                 scorer_hidden, dtype_code(kv_dtype))
         h = _P()
@@ -144,7 +150,8 @@ class KVpopCache:
         else:
             keep = [t.contiguous().float() for t in (W1, b1, w2, b2)]
             lg = None if log_gamma is None else log_gamma.contiguous().float()
-            sc = kvpop_scorer(*[t.data_ptr() for t in keep], None if lg is None else lg.data_ptr())
+            sc = kvpop_scorer(*[t.data_ptr() for t in keep], None if lg is None else lg.data_ptr(),
+                              1 if kv_only else 0, ACTIVATIONS[activation])
             _ck(kvpop_init_cache(ctypes.byref(self.cfg), ctypes.byref(sc), _stream(stream),
                                  ctypes.byref(h)), "kvpop_init_cache")
         self.handle = h.value

@@ -24,7 +24,8 @@ def make_cache(cfg, weights, mlstm=None):
     W1, b1, w2, b2, lg = weights
     return kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
                             cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
-                            log_gamma=(lg if cfg.log_gamma != 0.0 else None), n_sink=cfg.n_sink)
+                            log_gamma=(lg if cfg.log_gamma != 0.0 else None), n_sink=cfg.n_sink,
+                            activation=cfg.scorer_act, kv_only=cfg.scorer_kv_only)
 
 
 def injected_prefill_scores(cfg, Pmax, device, levels=None):

@@ -344,3 +344,35 @@ def test_pins_catch_planted_mistakes(monkeypatch):
     with pytest.raises(AssertionError):
         for z, phi in read_golden("normal_cdf.txt"):
             assert abs(ok.gelu_erf(float(z)) - float(z) * float(phi)) < 1e-12
+
+
+# ---------------------------------------------------------------- plain [k; v] scorer variants
+def test_silu_textbook_values():
+    """SiLU(z) = z * sigmoid(z); sigmoid(1) = 0.7310585786300049, sigmoid(2) = 0.8807970779778823."""
+    z = np.array([0.0, 1.0, 2.0, -1.0, -2.0, 60.0, -60.0])
+    want = [0.0, 0.7310585786300049, 2 * 0.8807970779778823, -(1 - 0.7310585786300049),
+            -2 * (1 - 0.8807970779778823), 60.0, 0.0]
+    got = ok.silu(z)
+    assert np.allclose(got, want, rtol=1e-14, atol=1e-24)
+
+
+@pytest.mark.parametrize("act", ["silu", "identity"])
+def test_kv_only_scorer_handset_weights(act):
+    """Input [k; v] (no query mean): W1 rows 0..d-1 read k, d..2d-1 read v."""
+    d, F, D = 2, 2, 2
+    W1 = np.zeros((2 * d, F))
+    W1[0, 0] = 1.0          # unit 0 <- k[0]
+    W1[d + 1, 1] = -2.0     # unit 1 <- -2 v[1]
+    b1 = np.array([0.5, 0.0])
+    w2 = np.array([1.0, 3.0])
+    p = OracleParams(W1, b1, w2, 0.25, 4, D, 0, 0.0, act)
+    c = HeadCache(p, d, 1)
+    k0, v0 = np.array([1.5, 9.0]), np.array([7.0, -0.75])
+    c.append(np.full((1, d), 100.0), k0, v0)
+    c.append(np.full((1, d), 100.0), np.zeros(d), np.zeros(d))
+    u, x = c.scorer_input(np.full(d, 100.0))
+    assert u == 0 and np.array_equal(x, np.concatenate([k0, v0]))
+    z0, z1 = 1.5 + 0.5, -2.0 * -0.75
+    f = ok.silu if act == "silu" else (lambda y: y)
+    want = 1.0 * f(z0) + 3.0 * f(z1) + 0.25
+    assert abs(float(ok.scorer_mlp(x, p)) - want) < 1e-14

@@ -33,6 +33,8 @@ class WorkloadConfig:
     n_layers: int = 1
     hidden: int = 0          # model width for the projection stack (layers > 1)
     seed: int = 0
+    scorer_act: str = "gelu"  # hidden activation of the stateless scorer: gelu / silu / identity
+    scorer_kv_only: bool = False  # scorer input [k; v] instead of [k; v; qbar]
     log_gamma: float = 0.0   # per-head log decay (0 = no decay)
     description: str = field(default="", compare=False)
 
@@ -46,7 +48,7 @@ class WorkloadConfig:
 
     @property
     def scorer_in(self) -> int:
-        return 3 * self.head_dim
+        return (2 if self.scorer_kv_only else 3) * self.head_dim
 
     def with_(self, **kw) -> "WorkloadConfig":
         return replace(self, **kw)
