@@ -8,6 +8,13 @@ compressed cache (kvpop_decode_attend).  Prefill is done once, untimed.
 
 Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle instead
 (the reference arm: the paper publishes no code and no decode throughput).
+
+``--workload prompt`` measures the prompt path instead (one step = one
+kvpop_prefill_attend call over a group of sequences: scoring, compression,
+static ranks, running top-k cutoffs and masked attention with outputs), and
+``--workload target`` the training target (one step = kvpop_future_target over
+the group, fed with the prompt pass's sparse normalisers).  Both print their
+own JSON line; the dominant kernel is tensor-bound.
 Under torchrun (N > 1) every rank runs an independent replica of the workload
 (the path has no cross-sequence exchange); value = all ranks' tokens / max time.
 """
@@ -49,6 +56,9 @@ def parse_args(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=96)
+    ap.add_argument("--workload", choices=["decode", "prompt", "target"], default="decode",
+                    help="decode steps (default), the prompt path with outputs, or the target pass")
+    ap.add_argument("--group", type=int, default=8, help="sequences per prompt/target step")
     return ap.parse_args(argv)
 
 
@@ -571,10 +581,268 @@ def run_reference(args):
     print(json.dumps(rec), flush=True)
 
 
+# ------------------------------------------------------------------ prompt path and target pass
+def measured_tensor_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured (MEASURED_PEAKS.json bf16_tflops, burst)"
+    return 1900.0, "fallback 1.9 PFLOP/s bf16 burst"
+
+
+def prompt_attention_flops(cfg, lengths) -> float:
+    """QK + PV flops of the masked prompt attention: 4 d G per retained (query, key)."""
+    import numpy as np
+    keep = cfg.budget_B + cfg.delay_D
+    tot = sum(int(np.minimum(np.arange(1, P + 1), keep).sum()) for P in lengths)
+    return 4.0 * cfg.head_dim * cfg.q_per_kv * cfg.n_kv_heads * tot
+
+
+def target_flops(cfg, lengths) -> float:
+    """QK flops of the transposed pass: 2 d G per (key t, future query d >= t + w)."""
+    import numpy as np
+    tot = 0
+    for P in lengths:
+        t = np.arange(P)
+        tot += int(np.maximum(0, P - t - cfg.delay_D).sum())
+    return 2.0 * cfg.head_dim * cfg.q_per_kv * cfg.n_kv_heads * tot
+
+
+def _oracle_prompt_job(args):
+    """Oracle time of one (sequence, KV head) prompt: scoring + compression, ranks and cutoffs
+    in full, masked attention on `nq` evenly spaced queries (extrapolated to all P)."""
+    cfg_name, b, h, nq, over = args
+    import numpy as np
+    import torch
+    torch.set_num_threads(1)
+    from oracle import running_topk as rt
+    from oracle.run import prefill_pair, _f64
+    from workload import gen, get_config
+    cfg = get_config(cfg_name, **over)
+    P = gen.prompt_lengths(cfg)[b]
+    G = cfg.q_per_kv
+    t0 = time.perf_counter()
+    cache = prefill_pair(cfg, gen.scorer_weights(cfg), b, h, P)
+    prio = rt.prompt_priorities(cache.prefill_raw, P, cfg.delay_D, cache.p.log_gamma)
+    rank = rt.static_ranks(prio)
+    tau = rt.fenwick_cutoffs(rank, cfg.n_sink, cfg.delay_D, cfg.budget_B - cfg.n_sink)
+    t_fixed = time.perf_counter() - t0
+    Q = _f64(gen.q_tokens(cfg, b, 1, 0, P, heads=range(h * G, (h + 1) * G)))[0]
+    K = _f64(gen.kv_tokens(cfg, "k", b, 1, 0, P, heads=[h]))[0, 0]
+    V = _f64(gen.kv_tokens(cfg, "v", b, 1, 0, P, heads=[h]))[0, 0]
+    qs = np.linspace(0, P - 1, nq).astype(int)
+    t0 = time.perf_counter()
+    for q in qs:
+        keys = np.nonzero(rt.mask_row(int(q), rank, tau, cfg.n_sink, cfg.delay_D))[0]
+        lg = Q[:, q, :] @ K[keys].T / np.sqrt(cfg.head_dim)
+        e = np.exp(lg - lg.max(axis=1, keepdims=True))
+        _ = (e / e.sum(axis=1, keepdims=True)) @ V[keys]
+    t_q = (time.perf_counter() - t0) / nq
+    return t_fixed + P * t_q
+
+
+def _oracle_target_job(args):
+    """Oracle time of one (sequence, KV head) target: the future log mass of `nk` evenly
+    spaced keys for every query head (extrapolated to all P keys)."""
+    cfg_name, b, h, nk, over = args
+    import numpy as np
+    import torch
+    torch.set_num_threads(1)
+    from oracle.run import _f64
+    from workload import gen, get_config
+    cfg = get_config(cfg_name, **over)
+    P = gen.prompt_lengths(cfg)[b]
+    G, d, w = cfg.q_per_kv, cfg.head_dim, cfg.delay_D
+    Q = _f64(gen.q_tokens(cfg, b, 1, 0, P, heads=range(h * G, (h + 1) * G)))[0]
+    K = _f64(gen.kv_tokens(cfg, "k", b, 1, 0, P, heads=[h]))[0, 0]
+    lse = np.zeros((G, P))            # normalisers are an input of the pass
+    ts = np.linspace(0, P - 1, nk).astype(int)
+    t0 = time.perf_counter()
+    for t in ts:
+        for g in range(G):
+            if t + w <= P - 1:
+                v = Q[g, t + w:] @ K[t] / np.sqrt(d) - lse[g, t + w:]
+                _ = np.logaddexp.reduce(v)
+    return (time.perf_counter() - t0) / nk * P
+
+
+def cpu_prompt_baseline(cfg, over, group, kind):
+    import multiprocessing as mp
+    cores = max(1, min(os.cpu_count() or 1, 16))
+    pairs = [(b % group, b % cfg.n_kv_heads) for b in range(cores)]
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+    ctx = mp.get_context("spawn")
+    job = _oracle_prompt_job if kind == "prompt" else _oracle_target_job
+    n = 48 if kind == "prompt" else 64
+    with ctx.Pool(len(pairs)) as pool:
+        times = pool.map(job, [(cfg.name, b, h, n, over) for b, h in pairs])
+    pair_s = statistics.mean(times)
+    group_s = group * cfg.n_kv_heads * pair_s / len(pairs)
+    what = ("scoring, compression, ranks and cutoffs in full plus masked attention of "
+            f"{n} evenly spaced queries" if kind == "prompt" else
+            f"future log mass of {n} evenly spaced keys for every query head")
+    return {"value": group * cfg.prompt_len / group_s, "unit": "tokens/s", "cores": len(pairs),
+            "kind": "oracle",
+            "sample": (f"{len(pairs)} (sequence, KV head) pairs of the {group}-sequence group, one "
+                       f"per core in parallel: {what}, extrapolated to the whole prompt and group")}
+
+
+def run_prompt_bench(args):
+    import torch
+    rank_, local_rank, world = dist_info()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = dist_init(world, "nccl")
+    from paper_2607_05061_gb300 import build as _build
+    _build.build()
+    from paper_2607_05061_gb300 import kvpop
+    from workload import gen, get_config
+    over = {}
+    if args.batch:
+        over["batch"] = args.batch
+    if args.prompt_len:
+        over["prompt_len"] = args.prompt_len
+    cfg = get_config(args.config, **over)
+    if cfg.n_layers != 1 or cfg.ragged:
+        raise SystemExit("--workload prompt/target runs fixed-length single-layer workloads")
+    n = min(args.group, cfg.batch)
+    P, H, G, d = cfg.prompt_len, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim
+    L = [P] * n
+    W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
+    cache = kvpop.KVpopCache(cfg.batch, H, G, d, cfg.budget_B, cfg.delay_D, cfg.scorer_hidden,
+                             cfg.kv_dtype, W1, b1, w2, b2, n_sink=cfg.n_sink)
+    Q = gen.q_tokens(cfg, 0, n, 0, P, device=dev)
+    K = gen.kv_tokens(cfg, "k", 0, n, 0, P, device=dev)
+    V = gen.kv_tokens(cfg, "v", 0, n, 0, P, device=dev)
+    Y = torch.empty((n, H * G, P, d), dtype=torch.float32, device=dev)
+    lse = torch.empty((n, H * G, P), dtype=torch.float32, device=dev)
+    rk = torch.empty((n, H, P), dtype=torch.int32, device=dev)
+    tu = torch.empty((n, H, P), dtype=torch.int32, device=dev)
+    logm = torch.empty((n, H * G, P), dtype=torch.float32, device=dev)
+    tgt = torch.empty((n, H, P), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    k_b = cfg.budget_B - cfg.n_sink
+
+    def prompt_step():
+        cache.prefill_attend(Q, K, V, L, Y, lse, rank=rk, tau=tu)
+
+    def target_step():
+        kvpop.future_target(Q, K, lse, cfg.delay_D, logm=logm, target=tgt)
+
+    def kernel_only():
+        if args.workload == "prompt":
+            kvpop.prompt_attention(Q, K, V, rk, tu, cfg.n_sink, cfg.delay_D, k_b, Y=Y, lse=lse)
+        else:
+            kvpop.future_target(Q, K, lse, cfg.delay_D, logm=logm, want_target=False)
+
+    step = prompt_step if args.workload == "prompt" else target_step
+    prompt_step()                                  # the target pass consumes these normalisers
+    W, Kn = max(3, args.warmup), args.steps
+    for _ in range(W):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(Kn):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    step_ms, _ = reduce_max_sum(e0.elapsed_time(e1) / Kn, 0.0, world, dev)
+    # dominant kernel alone (same stream, CUDA events)
+    ks = []
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        kernel_only()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ks.append(a.elapsed_time(b))
+    k_ms = statistics.mean(ks)
+    cache.check()
+    flops = prompt_attention_flops(cfg, L) if args.workload == "prompt" else target_flops(cfg, L)
+    peak, peak_src = measured_tensor_peak()
+    achieved = flops / (k_ms / 1e3) / 1e12
+    # end to end through the public API on pinned host buffers
+    Qh, Kh, Vh = Q.cpu().pin_memory(), K.cpu().pin_memory(), V.cpu().pin_memory()
+    if args.workload == "prompt":
+        outs_h = [torch.empty_like(Y, device="cpu").pin_memory(), torch.empty_like(lse, device="cpu").pin_memory()]
+        h2d = (Qh.numel() + Kh.numel() + Vh.numel()) * Qh.element_size()
+    else:
+        lse_h = lse.cpu().pin_memory()
+        outs_h = [torch.empty_like(tgt, device="cpu").pin_memory()]
+        h2d = (Qh.numel() + Kh.numel()) * Qh.element_size() + lse_h.numel() * 4
+    d2h = sum(o.numel() * o.element_size() for o in outs_h)
+    E = 2
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(E):
+        Q.copy_(Qh, non_blocking=True)
+        K.copy_(Kh, non_blocking=True)
+        if args.workload == "prompt":
+            V.copy_(Vh, non_blocking=True)
+            prompt_step()
+            outs_h[0].copy_(Y, non_blocking=True)
+            outs_h[1].copy_(lse, non_blocking=True)
+        else:
+            lse.copy_(lse_h, non_blocking=True)
+            target_step()
+            outs_h[0].copy_(tgt, non_blocking=True)
+        stream.synchronize()
+    e2e_s = (time.perf_counter() - t0) / E
+    tokens = n * P * world
+    if args.workload == "prompt":
+        metric = "prompt tokens/sec with outputs under the running top-k mask (1 GB300)"
+        kname = "prompt_tc_kernel" if cfg.kv_dtype == "bf16" else "prompt_simt_kernel"
+        what = ("kvpop_prefill_attend: delayed scorer on every prompt token, prompt compression, "
+                "static ranks + running top-k cutoffs, masked causal attention with y and LSE")
+    else:
+        metric = "future-target tokens/sec (transposed attention pass + aggregation, 1 GB300)"
+        kname = "target_tc_kernel" if cfg.kv_dtype == "bf16" else "target_simt_kernel"
+        what = ("kvpop_future_target with the prompt pass's sparse LSE: log future mass per key "
+                "and query head, max aggregation, count normalisation")
+    rec = {
+        "metric": metric, "value": tokens / (step_ms / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": Kn, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": cfg.kv_dtype,
+        "data": "synthetic (seeded counter-based generator)",
+        "config": {"workload": f"{cfg.name} prompt group: {n} sequences x {P} tokens, {H} KV heads "
+                               f"x {G} query heads, d {d}, B {cfg.budget_B}, D {cfg.delay_D}",
+                   "step": what,
+                   "l2": f"inputs larger than L2: Q/K/V {(Q.numel() + K.numel() + V.numel()) * 2 / 1e9:.2f} GB",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak,
+                     "peak_source": peak_src, "unit": "TFLOP/s", "frac": achieved / peak,
+                     "traffic": None, "algorithmic_flops_per_launch": flops, "ms_per_launch": k_ms},
+        "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": E,
+                "how": "pinned host inputs copied in, outputs copied out, inside the timed region"},
+        "gpu_launches": Kn * (5 if args.workload == "prompt" else 2),
+        "clocks": clk,
+    }
+    cache.free()
+    if rank_ == 0 and not args.no_cpu_baseline:
+        rec["cpu_baseline"] = cpu_prompt_baseline(cfg, over, n, args.workload)
+    if rank_ == 0:
+        print(json.dumps(rec), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload != "decode":
+        run_prompt_bench(args)
     else:
         run_kvpop(args)
 

@@ -22,169 +22,15 @@
 // V via ldmatrix.trans, probabilities packed to bf16 in registers), K/V rows
 // gathered by 16-byte cp.async into a 128-byte-swizzled double buffer.
 // fp32: CUDA-core kernel, one warp per (query, head) row, 32 keys per round.
-#include <climits>
+#include <cstdlib>
 
 #include "kvpop_mma.cuh"
+#include "kvpop_prompt.cuh"
 
 namespace kvpop {
 namespace {
 
-constexpr float kLn2 = 0.69314718055994530942f;
-
-struct PromptArgs {
-  const void* Q;             // [n_seq][H*G][S][d]
-  const void* K;             // [n_seq][H][S][d]
-  const void* V;
-  const int32_t* rank;       // [n_seq*H][S]
-  const int32_t* tau;        // [n_seq*H][S]
-  const int32_t* len;        // [n_seq] or nullptr (= S)
-  float* Y;                  // [n_seq][H*G][S][d]
-  float* lse;                // [n_seq][H*G][S] or nullptr
-  int H, G, S, s, w;
-  int capA, capM;
-  float qscale;              // log2(e) / sqrt(d)
-  int32_t* err;              // first-error word or nullptr
-};
-
-enum : int { PERR_LIST_OVERFLOW = 11 };
-
-__device__ __forceinline__ void note_err(int32_t* err, int code) {
-  if (err) atomicCAS(err, 0, code);
-}
-
-__device__ __forceinline__ bool keep_key(int q, int t, int r, int tq, int s, int w) {
-  return t <= q && (t < s || q - t < w || (t <= q - w && r <= tq));
-}
-
-// Shared prologue: tile bounds, per-query cutoffs, cutoff range, key lists.
-struct TileInfo {
-  int seq, h, pair, q0, q1, L;
-  int nA, nM;
-};
-
-template <int NT>
-__device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int32_t* posA,
-                           int32_t* posM, TileInfo& ti) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int NW = NT / 32;
-  ti.pair = blockIdx.y;
-  ti.seq = ti.pair / a.H;
-  ti.h = ti.pair - ti.seq * a.H;
-  ti.L = a.len ? max(0, min(a.len[ti.seq], a.S)) : a.S;
-  ti.q0 = (gridDim.x - 1 - blockIdx.x) * BM;        // longest tiles first
-  if (ti.q0 >= ti.L) return false;
-  ti.q1 = min(ti.q0 + BM - 1, ti.L - 1);
-  const int nq = ti.q1 - ti.q0 + 1;
-  const int32_t* tau = a.tau + (size_t)ti.pair * a.S;
-  const int32_t* rank = a.rank + (size_t)ti.pair * a.S;
-  for (int i = tid; i < BM; i += NT) tauS[i] = i < nq ? tau[ti.q0 + i] : -1;
-  __syncthreads();
-  if (warp == 0) {
-    int mn = INT_MAX, mx = INT_MIN;
-    for (int i = lane; i < nq; i += 32) {
-      mn = min(mn, tauS[i]);
-      mx = max(mx, tauS[i]);
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-      mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-      mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    }
-    if (lane == 0) {
-      red[NW] = mn;
-      red[NW + 1] = mx;
-    }
-  }
-  __syncthreads();
-  const int tmin = red[NW], tmax = red[NW + 1];
-  const int s = a.s, w = a.w, q0 = ti.q0, q1 = ti.q1;
-  // sinks
-  const int nAs = min(s, q0 + 1);
-  const int nMs = max(0, min(s, q1 + 1) - nAs);
-  for (int t = tid; t < nAs && t < a.capA; t += NT) posA[t] = t;
-  for (int j = tid; j < nMs && j < a.capM; j += NT) posM[j] = nAs + j;
-  int nA = nAs, nM = nMs;
-  // eligible for the whole tile: t in [s, q0 - w]
-  const int hi = q0 - w;
-  constexpr int EPT = 16;
-  if (hi >= s && tmax >= 0) {
-    for (int c0 = s; c0 <= hi; c0 += NT * EPT) {
-      const int t0 = c0 + tid * EPT;
-      int r[EPT];
-#pragma unroll
-      for (int e = 0; e < EPT; ++e) r[e] = (t0 + e <= hi) ? __ldg(rank + t0 + e) : INT_MAX;
-      int ca = 0, cm = 0;
-#pragma unroll
-      for (int e = 0; e < EPT; ++e) {
-        ca += r[e] <= tmin;
-        cm += (r[e] > tmin) & (r[e] <= tmax);
-      }
-      const int v = ca | (cm << 16);        // at most NT * EPT = 4096 per field
-      int x = v;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-      }
-      if (lane == 31) red[warp] = x;
-      __syncthreads();
-      int off = 0, tot = 0;
-#pragma unroll
-      for (int i = 0; i < NW; ++i) {
-        const int y = red[i];
-        if (i < warp) off += y;
-        tot += y;
-      }
-      const int ex = off + x - v;
-      int ia = nA + (ex & 0xffff), im = nM + (ex >> 16);
-#pragma unroll
-      for (int e = 0; e < EPT; ++e) {
-        if (r[e] <= tmin) {
-          if (ia < a.capA) posA[ia] = t0 + e;
-          ++ia;
-        } else if (r[e] <= tmax) {
-          if (im < a.capM) posM[im] = t0 + e;
-          ++im;
-        }
-      }
-      nA += tot & 0xffff;
-      nM += tot >> 16;
-      __syncthreads();
-    }
-  }
-  // window and newly eligible positions
-  const int c_lo = max(s, q0 - w + 1);
-  for (int t = c_lo + tid; t <= q1; t += NT) {
-    const int j = nM + (t - c_lo);
-    if (j < a.capM) posM[j] = t;
-  }
-  if (q1 >= c_lo) nM += q1 - c_lo + 1;
-  if (nA > a.capA || nM > a.capM) {
-    if (tid == 0) note_err(a.err, PERR_LIST_OVERFLOW);
-    nA = min(nA, a.capA);
-    nM = min(nM, a.capM);
-  }
-  ti.nA = nA;
-  ti.nM = nM;
-  __syncthreads();
-  return true;
-}
-
-// Dense causal tiles (no mask beyond causality): keys 0 .. q0 serve every query
-// of the tile (list A), q0 + 1 .. q1 only the later ones (list M); a key's
-// list index is its position.
-__device__ __forceinline__ bool dense_setup(const PromptArgs& a, int BM, TileInfo& ti) {
-  ti.pair = blockIdx.y;
-  ti.seq = ti.pair / a.H;
-  ti.h = ti.pair - ti.seq * a.H;
-  ti.L = a.len ? max(0, min(a.len[ti.seq], a.S)) : a.S;
-  ti.q0 = (gridDim.x - 1 - blockIdx.x) * BM;
-  if (ti.q0 >= ti.L) return false;
-  ti.q1 = min(ti.q0 + BM - 1, ti.L - 1);
-  ti.nA = ti.q0 + 1;
-  ti.nM = ti.q1 - ti.q0;
-  return true;
-}
+using namespace prompt;
 
 // ---------------------------------------------------------------- CUDA-core kernel
 constexpr int SIMT_NT = 256;
@@ -562,8 +408,27 @@ cudaError_t launch_simt(PromptArgs a, int n_pairs, cudaStream_t stream) {
   return launch_cfg(prompt_simt_kernel<T, HD, DENSE>, grid, SIMT_NT, smem, stream, a);
 }
 
+}  // namespace
+
+bool prompt_t5_ok(int d, int G, int s, int w, int k);
+cudaError_t launch_prompt_t5(const prompt::PromptArgs& a, int n_pairs, int G, bool dense,
+                             bool want_y, cudaStream_t stream);
+
+namespace {
+
+// tcgen05 kernel for bf16 with d = 128 (KVPOP_PROMPT_MMA_SYNC=1 selects the m16n8k16 kernel)
+bool use_t5(int dtype, int d, int G, int s, int w, int k) {
+  static const bool off = [] {
+    const char* e = getenv("KVPOP_PROMPT_MMA_SYNC");
+    return e && e[0] == '1';
+  }();
+  return !off && dtype == KVPOP_BF16 && prompt_t5_ok(d, G, s, w, k);
+}
+
 template <bool DENSE, bool WANT_Y>
 cudaError_t dispatch(const PromptArgs& a, int n_pairs, int dtype, int d, int G, cudaStream_t stream) {
+  if (use_t5(dtype, d, G, a.s, a.w, a.capA - a.s) && (DENSE || WANT_Y))
+    return launch_prompt_t5(a, n_pairs, G, DENSE, WANT_Y, stream);
   if (dtype == KVPOP_BF16) {
     if (d == 128) {
       if (G == 4) return launch_tc<128, 4, DENSE, WANT_Y>(a, n_pairs, stream);
