@@ -228,9 +228,14 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
             }
           }
         }
-        float mx = -INFINITY;
+        // 8 independent partial maxima (a 64-long chain would serialise on latency)
+        float pm[8];
 #pragma unroll
-        for (int i = 0; i < 64; ++i) mx = fmaxf(mx, s[i]);
+        for (int k = 0; k < 8; ++k) pm[k] = s[k];
+#pragma unroll
+        for (int i = 8; i < 64; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
+        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         const float mxs = mx * c2;                  // row maximum, log2 units
         float alpha = 1.f, m_new = m;
         bool resc = false;
@@ -240,8 +245,20 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
           resc = m != -INFINITY;
         }
         const float base = m_new == -INFINITY ? 0.f : m_new;
+        float ps[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          s[i] = ex2(fmaf(s[i], c2, -base));
+          ps[i & 7] += s[i];
+        }
+        const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        l = l * alpha + sum;
+        m = m_new;
         if (WANT_Y && j >= 1) {
-          // PV_{j-1} must have consumed the P tile (and landed in O) before it changes
+          // PV_{j-1} must have consumed the P tile (and landed in O) before either changes;
+          // the exponentials above overlap with it
           if (!(ok = uniform(mbar_wait(bar(B_ODONE + h), (j - 1) & 1, a.err, T5ERR_WAIT)))) break;
           if (__any_sync(0xffffffffu, resc)) {
             fence_after();
@@ -258,14 +275,6 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
             tmem_wait_st();
           }
         }
-        float sum = 0.f;
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          s[i] = ex2(fmaf(s[i], c2, -base));
-          sum += s[i];
-        }
-        l = l * alpha + sum;
-        m = m_new;
         if (WANT_Y) {
           unsigned char* prow = sm5 + L::OFF_P + h * PB;
 #pragma unroll
