@@ -211,6 +211,13 @@ kvpop_status kvpop_prompt_attention(const void* Q_dev, const void* K_dev, const 
                                     int32_t window, int32_t k, kvpop_dtype dtype, float* Y_dev,
                                     float* lse_dev, cudaStream_t stream);
 
+/* First device-side error (a bounded wait that expired) recorded by the
+ * cache-free calls kvpop_prompt_attention, kvpop_causal_lse and
+ * kvpop_future_target since the last call of this function: KVPOP_OK, or
+ * KVPOP_ERR_DEVICE_CHECK (details in kvpop_last_error).  Synchronises `stream`
+ * and clears the record. */
+kvpop_status kvpop_standalone_status(cudaStream_t stream);
+
 /* Dense causal log-normalisers (App. D.1), the exact-target variant of the
  * normaliser fed to kvpop_future_target:
  *   lse[q] = log sum_{t <= q} exp(q.k_t / sqrt(d))   per query head, natural log

@@ -40,7 +40,16 @@ struct kvpop_cache {
   uint64_t magic = 0;
 };
 
+// First device-side error of the cache-free calls (prompt attention, causal LSE,
+// future target); read and cleared by kvpop_standalone_status.
+__device__ int32_t g_standalone_err[4];
+
 namespace {
+
+int32_t* standalone_err() {
+  void* p = nullptr;
+  return cudaGetSymbolAddress(&p, g_standalone_err) == cudaSuccess ? static_cast<int32_t*>(p) : nullptr;
+}
 
 constexpr uint64_t kMagic = 0x6b7670'6f70'6361ull;   // "kvpopca"
 constexpr uint64_t kStateVersion = 1;
@@ -548,8 +557,8 @@ kvpop_status kvpop_prompt_attention(const void* Q, const void* K, const void* V,
       !aligned4(tau) || !aligned4(lengths) || !aligned4(lse))
     return KVPOP_ERR_ALIGN;
   cudaError_t e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, lengths, n_seq, n_kv_heads, q_per_kv,
-                                            head_dim, S, n_sink, window, k, dtype, Y, lse, nullptr,
-                                            stream));
+                                            head_dim, S, n_sink, window, k, dtype, Y, lse,
+                                            standalone_err(), stream));
   return from_cuda(e);
 }
 
@@ -563,7 +572,7 @@ kvpop_status kvpop_causal_lse(const void* Q, const void* K, const int32_t* lengt
   if (!Q || !K || !lse) return KVPOP_ERR_INVALID_ARG;
   if (!aligned16(Q) || !aligned16(K) || !aligned4(lse) || !aligned4(lengths)) return KVPOP_ERR_ALIGN;
   return from_cuda(NOTE(launch_causal_lse(Q, K, lengths, n_seq, n_kv_heads, q_per_kv, head_dim, S,
-                                          dtype, lse, stream)));
+                                          dtype, lse, standalone_err(), stream)));
 }
 
 kvpop_status kvpop_future_target(const void* Q, const void* K, const float* lse,
@@ -583,7 +592,23 @@ kvpop_status kvpop_future_target(const void* Q, const void* K, const float* lse,
     return KVPOP_ERR_ALIGN;
   return from_cuda(NOTE(launch_future_target(Q, K, lse, lengths, n_seq, n_kv_heads, q_per_kv,
                                              head_dim, S, window, lookahead, dtype, logm, target,
-                                             agg, count_norm, eps, stream)));
+                                             agg, count_norm, eps, standalone_err(), stream)));
+}
+
+kvpop_status kvpop_standalone_status(cudaStream_t stream) {
+  int32_t* d = standalone_err();
+  if (!d) return KVPOP_ERR_CUDA;
+  int32_t h = 0;
+  cudaError_t e = NOTE(cudaMemcpyAsync(&h, d, 4, cudaMemcpyDeviceToHost, stream));
+  if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
+  if (e != cudaSuccess) return from_cuda(e);
+  if (h != 0) {
+    std::snprintf(g_last_error, sizeof(g_last_error), "device error code %d", h);
+    e = NOTE(cudaMemsetAsync(d, 0, 4, stream));
+    if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
+    return e == cudaSuccess ? KVPOP_ERR_DEVICE_CHECK : from_cuda(e);
+  }
+  return KVPOP_OK;
 }
 
 kvpop_status kvpop_decode_ingest(kvpop_cache* c, const void* q, const void* k, const void* v,

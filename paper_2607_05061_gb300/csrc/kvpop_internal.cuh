@@ -140,12 +140,13 @@ cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, co
 
 // Dense causal log-normalisers of every prompt query (LSE only, no output rows).
 cudaError_t launch_causal_lse(const void* Q, const void* K, const int32_t* len, int n_seq, int H,
-                              int G, int d, int S, int dtype, float* lse, cudaStream_t stream);
+                              int G, int d, int S, int dtype, float* lse, int32_t* err,
+                              cudaStream_t stream);
 // Future-attention log masses (transposed pass) and the aggregated target.
 cudaError_t launch_future_target(const void* Q, const void* K, const float* lse, const int32_t* len,
                                  int n_seq, int H, int G, int d, int S, int w, int la, int dtype,
                                  float* logm, float* target, int agg, int count_norm, float eps,
-                                 cudaStream_t stream);
+                                 int32_t* err, cudaStream_t stream);
 
 // ------------------------------------------------------------------ device helpers
 __device__ __forceinline__ float to_f(float x) { return x; }

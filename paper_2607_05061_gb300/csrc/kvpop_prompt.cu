@@ -464,10 +464,11 @@ cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, co
 }
 
 cudaError_t launch_causal_lse(const void* Q, const void* K, const int32_t* len, int n_seq, int H,
-                              int G, int d, int S, int dtype, float* lse, cudaStream_t stream) {
+                              int G, int d, int S, int dtype, float* lse, int32_t* err,
+                              cudaStream_t stream) {
   if (n_seq <= 0 || S <= 0) return cudaSuccess;
   PromptArgs a{Q, K, nullptr, nullptr, nullptr, len, nullptr, lse, H, G, S, 0, 1, 0, 0,
-               1.4426950408889634f / sqrtf((float)d), nullptr};
+               1.4426950408889634f / sqrtf((float)d), err};
   return dispatch<true, false>(a, n_seq * H, dtype, d, G, stream);
 }
 

@@ -40,14 +40,14 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Bounded wait: false (and an error code recorded) after kWaitLimitNs.
+// Bounded wait: false (and an error code recorded in *err, if given) after kWaitLimitNs.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t* err, int code) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   for (unsigned it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0u && globaltimer() - t0 > kWaitLimitNs) {
-      atomicCAS(err, 0, code);
+      if (err) atomicCAS(err, 0, code);
       return false;
     }
   }

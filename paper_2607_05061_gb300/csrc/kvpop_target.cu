@@ -13,11 +13,23 @@
 // value output of the pass is never formed.  bf16 on m16n8k16 tensor-core
 // MMAs, fp32 on CUDA cores (one warp per (key, head), 32 queries per round).
 //
+// bf16 with d = 128 runs on the 5th-generation tensor cores (target_t5_kernel):
+// a CTA holds 256 keys as two 128-row A tiles in shared memory; producer warps
+// stream each head's query rows in blocks of 64 (with their LSE_d) through an
+// 8-stage cp.async ring; one thread issues S = K Q^T per half into a
+// tensor-memory double buffer; one softmax thread per (key, half) reads its row
+// with 32x32b loads and keeps the running max and sum.  The query rows are
+// contiguous, so the ring can run deep; the pass has no value half.
+//
 // Kernel 2 aggregates per KV head (Eq. 2, App. F.1-F.2):
 //   r_t = log(eps + Agg_g mbar_t^(g) / N_t),  N_t = max(1, S - (t + w)),
 // N_t clipped to L + 1 with a lookahead, Agg = max or mean; without count
 // normalisation N_t = 1.
+#include <cstdlib>
+
 #include "kvpop_mma.cuh"
+#include "kvpop_ptx.cuh"
+#include "kvpop_tc05.cuh"
 
 namespace kvpop {
 namespace {
@@ -33,6 +45,7 @@ struct TargetArgs {
   float* logm;               // [n][H*G][S] out
   int H, G, S, w, la;
   float kscale;              // log2(e) / sqrt(d)
+  int32_t* err;              // first-error word or nullptr
 };
 
 __device__ __forceinline__ int row_len(const TargetArgs& a, int seq) {
@@ -268,6 +281,187 @@ __global__ void __launch_bounds__(TgP<HD>::THREADS, 1) target_tc_kernel(TargetAr
   cp_wait<0>();
 }
 
+// ---------------------------------------------------------------- tcgen05 kernel (d = 128)
+constexpr int T6_HALF = 128;
+constexpr int T6_ROWS = 2 * T6_HALF;            // keys per CTA
+constexpr int T6_BN = 64;                       // queries per block
+constexpr int T6_ST = 8;                        // query-block stages
+constexpr int T6_MMA_WARP = 8;                  // warps 0-7 softmax, 8 MMA, 9-11 producers
+constexpr int T6_PT = 96;
+constexpr int T6_THREADS = 32 * 12;
+constexpr int T6_KB = T6_HALF * 256;            // key tile of one half
+constexpr int T6_QB = T6_BN * 256;              // query block
+constexpr int T6_OFF_Q = 2 * T6_KB;
+constexpr int T6_OFF_LSE = T6_OFF_Q + T6_ST * T6_QB;
+constexpr int T6_OFF_BAR = T6_OFF_LSE + T6_ST * T6_BN * 4;
+constexpr int T6_OFF_TMEM = T6_OFF_BAR + 8 * 32;
+constexpr int T6_SMEM = T6_OFF_TMEM + 16;
+constexpr int T6_FULL = 0, T6_EMPTY = T6_ST, T6_SFULL = 2 * T6_ST, T6_PFULL = 2 * T6_ST + 4,
+              T6_KFULL = 2 * T6_ST + 8;
+enum : int { T6ERR_WAIT = 22 };
+
+template <int G>
+__global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) {
+  using namespace tc05;
+  extern __shared__ __align__(1024) unsigned char sm6[];
+  const uint32_t sb = smem_u32(sm6);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int pair = blockIdx.y, seq = pair / a.H, h0 = pair - seq * a.H;
+  const int S = a.S, L = row_len(a, seq), w = a.w, la = a.la;
+  const int t0 = blockIdx.x * T6_ROWS;
+  if (t0 >= L) return;
+  const int t1 = min(t0 + T6_ROWS - 1, L - 1);
+  const size_t qrow0 = (size_t)seq * a.H * G + (size_t)h0 * G;
+  const int d_lo = t0 + w;
+  const int d_hi = la > 0 ? min(L - 1, t1 + w + la) : L - 1;
+  if (d_lo > d_hi) {                               // no key of the tile has a future query
+    for (int i = tid; i < (t1 - t0 + 1) * G; i += T6_THREADS) {
+      const int tl = i / G, g = i - tl * G;
+      a.logm[(qrow0 + g) * S + t0 + tl] = -INFINITY;
+    }
+    return;
+  }
+  const int nblk = (d_hi - d_lo + T6_BN) / T6_BN;
+  const int total = G * nblk;
+  auto bar = [&](int i) { return sb + T6_OFF_BAR + 8u * (uint32_t)i; };
+  if (tid == 0) {
+    for (int i = 0; i < T6_ST; ++i) {
+      mbar_init(bar(T6_FULL + i), T6_PT);
+      mbar_init(bar(T6_EMPTY + i), 1 + 2 * T6_HALF);   // MMA commit + every softmax thread (LSE)
+    }
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(bar(T6_SFULL + i), 1);
+      mbar_init(bar(T6_PFULL + i), T6_HALF);
+    }
+    mbar_init(bar(T6_KFULL), T6_PT);
+    mbar_fence_init();
+  }
+  if (warp == T6_MMA_WARP) tmem_alloc(sb + T6_OFF_TMEM, 256);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(sm6 + T6_OFF_TMEM);
+  const bf16* Kp = static_cast<const bf16*>(a.K) + (size_t)pair * S * 128;
+  if (warp > T6_MMA_WARP) {
+    // ---------------------------------------------------------------- producers
+    const int pt = tid - 32 * (T6_MMA_WARP + 1);
+    for (int i = pt; i < T6_ROWS * 16; i += T6_PT) {
+      const int r = i >> 4, c = i & 15;
+      const bool ok = t0 + r <= t1;
+      cp_async16(sb + (r >> 7) * T6_KB + tile_off(r & 127, c, T6_HALF),
+                 Kp + (size_t)(ok ? t0 + r : t0) * 128 + c * 8, ok ? 16 : 0);
+    }
+    cp_async_arrive_noinc(bar(T6_KFULL));
+    for (int j = 0; j < total; ++j) {
+      const int st = j % T6_ST;
+      if (j >= T6_ST && !mbar_wait(bar(T6_EMPTY + st), ((j / T6_ST) - 1) & 1, a.err, T6ERR_WAIT)) break;
+      const int g = j / nblk, b = j - g * nblk;
+      const int d0 = d_lo + b * T6_BN;
+      const bf16* Qg = static_cast<const bf16*>(a.Q) + (qrow0 + g) * S * 128;
+      const uint32_t qd = sb + T6_OFF_Q + st * T6_QB;
+      for (int i = pt; i < T6_BN * 16; i += T6_PT) {
+        const int r = i >> 4, c = i & 15;
+        const bool ok = d0 + r <= d_hi;
+        cp_async16(qd + tile_off(r, c, T6_BN), Qg + (size_t)(ok ? d0 + r : d0) * 128 + c * 8, ok ? 16 : 0);
+      }
+      if (pt < T6_BN) {
+        const float* lse = a.lse + (qrow0 + g) * S;
+        cp_async4(sb + T6_OFF_LSE + (st * T6_BN + pt) * 4, lse + min(d0 + pt, d_hi));
+      }
+      cp_async_arrive_noinc(bar(T6_FULL + st));
+    }
+    cp_wait<0>();
+  } else if (warp == T6_MMA_WARP) {
+    // ---------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      const uint32_t idS = idesc_bf16(128, T6_BN, 0);
+      bool ok = mbar_wait(bar(T6_KFULL), 0, a.err, T6ERR_WAIT);
+      for (int j = 0; j < total && ok; ++j) {
+        const int st = j % T6_ST, b2 = j & 1;
+        if (!(ok = mbar_wait(bar(T6_FULL + st), (j / T6_ST) & 1, a.err, T6ERR_WAIT))) break;
+        fence_async_smem();
+        fence_after();
+        const uint32_t qb = sb + T6_OFF_Q + st * T6_QB;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          // the softmax half must be done with S_{j-2} before its buffer is rewritten
+          if (j >= 2 && !(ok = mbar_wait(bar(T6_PFULL + 2 * hh + b2), ((j - 2) >> 1) & 1, a.err, T6ERR_WAIT)))
+            break;
+          fence_after();
+          const uint32_t dS = tmem + hh * 128 + (uint32_t)b2 * T6_BN;
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks)
+            mma_bf16(dS, kmajor_desc(sb + hh * T6_KB, T6_HALF, ks), kmajor_desc(qb, T6_BN, ks), idS, ks > 0);
+          commit(bar(T6_SFULL + 2 * hh + b2));
+        }
+        if (!ok) break;
+        commit(bar(T6_EMPTY + st));
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------------------------------------------------------- softmax rows
+    const int hh = warp >> 2;
+    const int r = (warp & 3) * 32 + lane;
+    const int t = t0 + hh * T6_HALF + r;
+    const int hi = t <= t1 ? future_hi(t, L, w, la) : -1;
+    const uint32_t tS = tmem + ((uint32_t)((warp & 3) * 32) << 16) + hh * 128;
+    const float* lseS = reinterpret_cast<const float*>(sm6 + T6_OFF_LSE);
+    const float c2 = a.kscale;
+    float m = -INFINITY, l = 0.f;
+    auto uniform = [](bool x) { return __all_sync(0xffffffffu, x); };
+    for (int j = 0; j < total; ++j) {
+      const int st = j % T6_ST, b2 = j & 1;
+      const int g = j / nblk, b = j - g * nblk;
+      const int d0 = d_lo + b * T6_BN;
+      if (!uniform(mbar_wait(bar(T6_SFULL + 2 * hh + b2), (j >> 1) & 1, a.err, T6ERR_WAIT))) break;
+      fence_after();
+      float s[64];
+      tmem_ld32(tS + b2 * T6_BN, *reinterpret_cast<float(*)[32]>(s));
+      tmem_ld32(tS + b2 * T6_BN + 32, *reinterpret_cast<float(*)[32]>(s + 32));
+      tmem_wait_ld();
+      // the stage's query rows and LSE are no longer needed once read
+#pragma unroll
+      for (int i = 0; i < 64; ++i) s[i] = fmaf(s[i], c2, -lseS[st * T6_BN + i] * kLog2e);
+      fence_before();
+      mbar_arrive(bar(T6_EMPTY + st));
+      mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
+      const bool masked = d0 < t1 + w || d0 + T6_BN - 1 > d_hi || (la > 0 && d0 + T6_BN - 1 > t0 + w + la);
+      if (masked) {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          const int d = d0 + i;
+          if (d < t + w || d > hi) s[i] = -INFINITY;
+        }
+      }
+      float pm[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) pm[k] = s[k];
+#pragma unroll
+      for (int i = 8; i < 64; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      const float mn = fmaxf(m, mx);
+      const float base = mn == -INFINITY ? 0.f : mn;
+      float ps[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+#pragma unroll
+      for (int i = 0; i < 64; ++i) ps[i & 7] += ex2(s[i] - base);
+      l = l * ex2(m - base) + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
+      m = mn;
+      if (b == nblk - 1) {                          // head g done: write and reset
+        if (t <= t1) a.logm[(qrow0 + g) * S + t] = l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
+        m = -INFINITY;
+        l = 0.f;
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == T6_MMA_WARP) tmem_dealloc(tmem, 256);
+}
+
 // ---------------------------------------------------------------- aggregation
 struct AggArgs {
   const float* logm;         // [n][H*G][S]
@@ -314,11 +508,29 @@ __global__ void aggregate_kernel(AggArgs a) {
 cudaError_t launch_future_target(const void* Q, const void* K, const float* lse, const int32_t* len,
                                  int n_seq, int H, int G, int d, int S, int w, int la, int dtype,
                                  float* logm, float* target, int agg, int count_norm, float eps,
-                                 cudaStream_t stream) {
+                                 int32_t* err, cudaStream_t stream) {
   if (n_seq <= 0 || S <= 0) return cudaSuccess;
-  TargetArgs a{Q, K, lse, len, logm, H, G, S, w, la, 1.4426950408889634f / sqrtf((float)d)};
+  TargetArgs a{Q, K, lse, len, logm, H, G, S, w, la, 1.4426950408889634f / sqrtf((float)d), err};
   const int n_pairs = n_seq * H;
-  if (dtype == KVPOP_BF16) {
+  static const bool mma_sync = [] {
+    const char* e = getenv("KVPOP_TARGET_MMA_SYNC");
+    return e && e[0] == '1';
+  }();
+  if (dtype == KVPOP_BF16 && d == 128 && !mma_sync) {
+    dim3 grid((S + T6_ROWS - 1) / T6_ROWS, n_pairs);
+    cudaError_t e = cudaSuccess;
+    if (G == 4) {
+      e = cudaFuncSetAttribute(target_t5_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      if (e == cudaSuccess) target_t5_kernel<4><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
+    } else if (G == 2) {
+      e = cudaFuncSetAttribute(target_t5_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      if (e == cudaSuccess) target_t5_kernel<2><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
+    } else {
+      e = cudaFuncSetAttribute(target_t5_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      if (e == cudaSuccess) target_t5_kernel<1><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
+    }
+    if (e != cudaSuccess) return e;
+  } else if (dtype == KVPOP_BF16) {
     const size_t smem = d == 128 ? TgP<128>::SMEM : TgP<64>::SMEM;
     dim3 grid((S + TgP<128>::ROWS - 1) / TgP<128>::ROWS, n_pairs);
     if (d == 128) {

@@ -81,6 +81,7 @@ _SIGS = {
     "kvpop_future_target": (ctypes.c_int, [_P, _P, _P, _P, c_int32, c_int32, c_int32, c_int32, c_int32,
                                            c_int32, c_int32, ctypes.c_int, _P, _P, c_int32, c_int32,
                                            c_float, _P]),
+    "kvpop_standalone_status": (ctypes.c_int, [_P]),
     "kvpop_last_error": (ctypes.c_char_p, []),
     "kvpop_debug_fail_alloc_after": (None, [c_int32]),
 }
