@@ -8,16 +8,22 @@
 // histogram pass up front gives every pass its bucket bases.  The last pass
 // writes rank[position] directly.
 //
-// Kernel 2 (one warp per row) computes tau_q for every query position.  The
-// paper inserts each newly eligible rank into a Fenwick tree and reads the k-th
-// smallest by binary lifting.  Here the same value comes from the observation
+// Kernel 2 (one CTA per row, the queries split into up to 16 chunks, one warp
+// each) computes tau_q for every query position.  The paper inserts each newly
+// eligible rank into a Fenwick tree and reads the k-th smallest by binary
+// lifting.  Here the same value comes from the observation
 // that tau_q never increases once k tokens are eligible: a bitset over ranks
 // (8 KB for 65536 tokens, in shared memory) marks the inserted ranks, and when a
 // newcomer ranks below the current cutoff the cutoff steps down to the next
 // marked rank below it -- the warp scans 32 bitset words per ballot.  Over a
 // whole row the cutoff moves down at most S ranks, so the scan is O(S) words
-// plus O(1) per query.  While fewer than k tokens are eligible every one of
-// them is kept, so tau_q is the largest inserted rank (-1 while none is).
+// plus O(1) per query.  A chunk's warp starts from the state the scan would have
+// reached: it marks the ranks of the tokens already eligible and takes the
+// min(k, n)-th marked rank as the cutoff (a popcount prefix over the bitset).
+// While fewer than k tokens are eligible every one of them is kept, so tau_q is
+// the largest inserted rank (-1 while none is).
+#include <algorithm>
+
 #include "kvpop_internal.cuh"
 
 namespace kvpop {
@@ -25,7 +31,7 @@ namespace {
 
 constexpr int RK_NT = 512;
 constexpr int RK_NW = RK_NT / 32;
-constexpr int CUT_WARPS = 4;
+constexpr int CUT_MAX_WARPS = 16;
 
 struct RankArgs {
   const float* prio;         // [n_rows][S]
@@ -179,26 +185,81 @@ __device__ __forceinline__ int marked_below(const uint32_t* bits, int r, int lan
   return -1;
 }
 
-__global__ void __launch_bounds__(CUT_WARPS * 32) cutoff_kernel(CutArgs a) {
+// Smallest marked rank whose count of marked ranks at or below it reaches c
+// (c >= 1 and at least c ranks marked); warp-collective.
+__device__ __forceinline__ int kth_marked(const uint32_t* bits, int words, int c, int lane) {
+  int base = 0;
+  for (int w0 = 0; w0 < words; w0 += 32) {
+    const int wi = w0 + lane;
+    const uint32_t v = wi < words ? bits[wi] : 0u;
+    const int cnt = __popc(v);
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    if (base + total >= c) {
+      const uint32_t hit = __ballot_sync(0xffffffffu, base + incl >= c);
+      const int l = __ffs(hit) - 1;
+      uint32_t word = __shfl_sync(0xffffffffu, v, l);
+      int need = c - (base + __shfl_sync(0xffffffffu, incl - cnt, l));
+      int bit = 0;
+      for (; bit < 32; ++bit) {
+        if ((word >> bit) & 1u) {
+          if (--need == 0) break;
+        }
+      }
+      return (w0 + l) * 32 + bit;
+    }
+    base += total;
+  }
+  return -1;
+}
+
+// One CTA per row; warp c takes the queries [c * chunk, (c + 1) * chunk).  It first
+// rebuilds the state the scan has just before its first query -- the bitset of
+// the ranks inserted so far and the cutoff, the min(k, n)-th smallest of them --
+// then runs the same per-query update, so every chunk's cutoffs equal those of
+// one scan over the whole row.
+__global__ void cutoff_kernel(CutArgs a, int chunk) {
   extern __shared__ uint32_t bitsets[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int row = blockIdx.x * CUT_WARPS + warp;
-  if (row >= a.n_rows) return;
+  const int row = blockIdx.x;
   const int S = a.S, words = (S + 31) >> 5;
-  uint32_t* bits = bitsets + (size_t)warp * words;
-  for (int i = lane; i < words; i += 32) bits[i] = 0u;
-  __syncwarp();
   const int L = row_length(a.len, a.rows_per_len, row, S);
   const int32_t* rank = a.rank + (size_t)row * S;
   int32_t* tau_out = a.tau + (size_t)row * S;
+  if (warp == 0)
+    for (int i = L + lane; i < S; i += 32) tau_out[i] = -1;
+  const int qa = warp * chunk;
+  if (qa >= L) return;
+  const int qb = min(qa + chunk, L);
+  uint32_t* bits = bitsets + (size_t)warp * words;
+  for (int i = lane; i < words; i += 32) bits[i] = 0u;
+  __syncwarp();
   const int s = a.s, w = a.w, k = a.k;
-  int tau = -1, n = 0;
-  for (int q0 = 0; q0 < L; q0 += 32) {
+  // tokens inserted before query qa: positions s .. qa - 1 - w
+  int cnt = 0;
+  for (int t = s + lane; t <= qa - 1 - w; t += 32) {
+    const int r = rank[t];
+    if (r >= 0 && r < S) {
+      atomicOr(&bits[r >> 5], 1u << (r & 31));
+      ++cnt;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  __syncwarp();
+  int n = cnt;
+  int tau = n > 0 ? kth_marked(bits, words, min(k, n), lane) : -1;
+  for (int q0 = qa; q0 < qb; q0 += 32) {
     const int tl = q0 + lane - w;
     int r_l = -1;
     if (tl >= s && tl < L) r_l = rank[tl];
     int mine = -1;
-    const int nq = min(32, L - q0);
+    const int nq = min(32, qb - q0);
     for (int j = 0; j < nq; ++j) {
       const int t = q0 + j - w;
       if (t >= s) {
@@ -215,7 +276,6 @@ __global__ void __launch_bounds__(CUT_WARPS * 32) cutoff_kernel(CutArgs a) {
     }
     if (lane < nq) tau_out[q0 + lane] = mine;
   }
-  for (int i = L + lane; i < S; i += 32) tau_out[i] = -1;
 }
 
 }  // namespace
@@ -238,13 +298,15 @@ cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len,
   rank_kernel<<<n_rows, RK_NT, 0, stream>>>(ra);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const size_t smem = (size_t)CUT_WARPS * ((S + 31) / 32) * 4;
-  if (smem > 48 * 1024) {
-    e = cudaFuncSetAttribute(cutoff_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
+  // chunks per row: up to 16 warps, each with its own bitset of S bits in shared memory
+  const size_t words_bytes = (size_t)((S + 31) / 32) * 4;
+  const int nch = (int)std::max<size_t>(1, std::min<size_t>(CUT_MAX_WARPS, (200 * 1024) / words_bytes));
+  const int chunk = (S + nch - 1) / nch;
+  const size_t smem = (size_t)nch * words_bytes;
+  e = cudaFuncSetAttribute(cutoff_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   CutArgs ca{rank, len, rows_per_len, n_rows, S, s, w, k, tau};
-  cutoff_kernel<<<(n_rows + CUT_WARPS - 1) / CUT_WARPS, CUT_WARPS * 32, smem, stream>>>(ca);
+  cutoff_kernel<<<n_rows, nch * 32, smem, stream>>>(ca, chunk);
   return cudaGetLastError();
 }
 
