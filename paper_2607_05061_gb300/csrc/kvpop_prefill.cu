@@ -13,6 +13,8 @@
 // on the order-preserving bit pattern of the fp32 priority, ties resolved by
 // position -- writes them to slots 0.. in ascending position, and loads the
 // window with the last min(P, D) tokens.
+#include <algorithm>
+
 #include "kvpop_argmin.cuh"
 
 namespace kvpop {
@@ -161,6 +163,203 @@ __global__ void __launch_bounds__(NT1) prefill_score_kernel(ScoreArgs<T> a) {
       const float rr = canon_score(s + a.st.b2[h]);
       prio_out[u] = static_priority(rr, u, a.st.log_gamma, h);
     }
+  }
+}
+
+// Register-tiled version for F in {128, 256}: a CTA scores UT2 = 64 consecutive
+// tokens; the scorer inputs X [3d][64] sit in shared memory (fp32, rows padded
+// to 68 floats), W1 streams
+// through in chunks of 32 input rows (double-buffered cp.async), and each thread
+// accumulates 4 tokens x NH hidden units (NH = F / 16), so every W1 row loaded
+// serves 64 tokens and every shared-memory read feeds 4 NH multiply-adds.
+constexpr int UT2 = 64;
+constexpr int XS2 = UT2 + 4;       // row stride of X in shared memory (float4-aligned, few bank conflicts)
+constexpr int KC2 = 32;
+constexpr int NT3 = 256;
+
+template <int NH>
+__host__ __device__ constexpr int gemm_w_bytes() { return 2 * KC2 * 16 * NH * 4; }
+
+template <typename T, int NH>
+__global__ void __launch_bounds__(NT3) prefill_score_gemm_kernel(ScoreArgs<T> a) {
+  constexpr int F = 16 * NH;
+  const Dims& dm = a.dm;
+  const int d = dm.d, D = dm.D, G = dm.G, H = dm.H;
+  const int lp = blockIdx.y;
+  const int bl = lp / H, h = lp - bl * H;
+  const int P = a.plen[bl];
+  const int n_elig = max(P - D, 0);
+  const int u0 = blockIdx.x * UT2;
+  if (u0 >= n_elig) return;
+  const int nrow = min(UT2, n_elig - u0);
+  const size_t Pm = a.Pmax;
+  const int tid = threadIdx.x;
+  const int in_dim = 3 * d;
+
+  extern __shared__ __align__(16) unsigned char smem[];
+  float* Xs = reinterpret_cast<float*>(smem);                    // [3d][XS2]
+  float* Wc = Xs + (size_t)in_dim * XS2;                          // [2][KC2][F]; staging first
+  const T* Kp = a.K + ((size_t)bl * H + h) * Pm * d;
+  const T* Vp = a.V + ((size_t)bl * H + h) * Pm * d;
+  const T* Qp = a.Q + ((size_t)bl * H * G + (size_t)h * G) * Pm * d;
+
+  // Staging with 16-byte loads, NB items per thread issued before any is used.
+  constexpr int CE = 16 / (int)sizeof(T);         // elements per 16-byte chunk
+  constexpr int NB = 4;
+  const int cpr = d / CE;                         // chunks per row
+  auto unpack = [](const uint4& v, float (&f)[CE]) {
+    const T* e = reinterpret_cast<const T*>(&v);
+#pragma unroll
+    for (int k = 0; k < CE; ++k) f[k] = to_f(e[k]);
+  };
+  // k_u, v_u -> X rows 0..2d-1 (transposed: X[channel][token])
+  for (int base = tid; base < UT2 * cpr; base += NT3 * NB) {
+    uint4 kk[NB], vv[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const int it = base + b * NT3;
+      const int r = it / cpr, c = it - r * cpr;
+      kk[b] = vv[b] = make_uint4(0u, 0u, 0u, 0u);
+      if (it < UT2 * cpr && r < nrow) {
+        kk[b] = __ldg(reinterpret_cast<const uint4*>(Kp + (size_t)(u0 + r) * d) + c);
+        vv[b] = __ldg(reinterpret_cast<const uint4*>(Vp + (size_t)(u0 + r) * d) + c);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const int it = base + b * NT3;
+      if (it >= UT2 * cpr) break;
+      const int r = it / cpr, c = it - r * cpr;
+      float fk[CE], fv[CE];
+      unpack(kk[b], fk);
+      unpack(vv[b], fv);
+#pragma unroll
+      for (int k = 0; k < CE; ++k) {
+        Xs[(c * CE + k) * XS2 + r] = fk[k];
+        Xs[(d + c * CE + k) * XS2 + r] = fv[k];
+      }
+    }
+  }
+  // query means of positions u0+1 .. u0+nrow-1+D, then qbar_u = mean of the D after u
+  float* qm = Wc;                                                  // [UT2 + D - 1][d]
+  const int npos = nrow - 1 + D;
+  for (int base = tid; base < npos * cpr; base += NT3 * NB) {
+    float acc[NB][CE];
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+#pragma unroll
+      for (int k = 0; k < CE; ++k) acc[b][k] = 0.f;
+    for (int g = 0; g < G; ++g) {
+      uint4 qv[NB];
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        const int it = base + b * NT3;
+        const int tt = it / cpr, c = it - tt * cpr;
+        qv[b] = make_uint4(0u, 0u, 0u, 0u);
+        if (it < npos * cpr)
+          qv[b] = __ldg(reinterpret_cast<const uint4*>(Qp + ((size_t)g * Pm + u0 + 1 + tt) * d) + c);
+      }
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        float f[CE];
+        unpack(qv[b], f);
+#pragma unroll
+        for (int k = 0; k < CE; ++k) acc[b][k] += f[k];
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const int it = base + b * NT3;
+      if (it >= npos * cpr) break;
+      const int tt = it / cpr, c = it - tt * cpr;
+#pragma unroll
+      for (int k = 0; k < CE; ++k) qm[tt * d + c * CE + k] = acc[b][k] * (1.0f / (float)G);
+    }
+  }
+  __syncthreads();
+  for (int idx = tid; idx < UT2 * d; idx += NT3) {
+    const int r = idx / d, i = idx - r * d;
+    float acc = 0.f;
+    if (r < nrow)
+      for (int j = 0; j < D; ++j) acc += qm[(r + j) * d + i];
+    Xs[(2 * d + i) * XS2 + r] = r < nrow ? acc / (float)D : 0.f;
+  }
+  __syncthreads();
+
+  const float* W1 = a.st.W1 + (size_t)h * in_dim * dm.Fp;       // Fp == F on this path
+  const uint32_t wbase = (uint32_t)__cvta_generic_to_shared(Wc);
+  auto load_chunk = [&](int c, int buf) {
+    const float* src = W1 + (size_t)c * KC2 * F;
+    for (int i = tid; i < KC2 * F / 4; i += NT3)
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(wbase + (uint32_t)((buf * KC2 * F + i * 4) * 4)),
+                   "l"(src + i * 4)
+                   : "memory");
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  const int tm = tid & 15, tn = tid >> 4;
+  float acc[4][NH];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int f = 0; f < NH; ++f) acc[r][f] = 0.f;
+  const int nchunk = in_dim / KC2;
+  load_chunk(0, 0);
+  for (int c = 0; c < nchunk; ++c) {
+    if (c + 1 < nchunk) {
+      load_chunk(c + 1, (c + 1) & 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();
+    const float* wb = Wc + (c & 1) * KC2 * F + tn * NH;
+    const float* xb = Xs + (size_t)c * KC2 * XS2 + tm * 4;
+#pragma unroll 4
+    for (int kk = 0; kk < KC2; ++kk) {
+      const float4 x = *reinterpret_cast<const float4*>(xb + kk * XS2);
+#pragma unroll
+      for (int f4 = 0; f4 < NH / 4; ++f4) {
+        const float4 w = *reinterpret_cast<const float4*>(wb + kk * F + f4 * 4);
+        acc[0][4 * f4 + 0] = fmaf(x.x, w.x, acc[0][4 * f4 + 0]);
+        acc[0][4 * f4 + 1] = fmaf(x.x, w.y, acc[0][4 * f4 + 1]);
+        acc[0][4 * f4 + 2] = fmaf(x.x, w.z, acc[0][4 * f4 + 2]);
+        acc[0][4 * f4 + 3] = fmaf(x.x, w.w, acc[0][4 * f4 + 3]);
+        acc[1][4 * f4 + 0] = fmaf(x.y, w.x, acc[1][4 * f4 + 0]);
+        acc[1][4 * f4 + 1] = fmaf(x.y, w.y, acc[1][4 * f4 + 1]);
+        acc[1][4 * f4 + 2] = fmaf(x.y, w.z, acc[1][4 * f4 + 2]);
+        acc[1][4 * f4 + 3] = fmaf(x.y, w.w, acc[1][4 * f4 + 3]);
+        acc[2][4 * f4 + 0] = fmaf(x.z, w.x, acc[2][4 * f4 + 0]);
+        acc[2][4 * f4 + 1] = fmaf(x.z, w.y, acc[2][4 * f4 + 1]);
+        acc[2][4 * f4 + 2] = fmaf(x.z, w.z, acc[2][4 * f4 + 2]);
+        acc[2][4 * f4 + 3] = fmaf(x.z, w.w, acc[2][4 * f4 + 3]);
+        acc[3][4 * f4 + 0] = fmaf(x.w, w.x, acc[3][4 * f4 + 0]);
+        acc[3][4 * f4 + 1] = fmaf(x.w, w.y, acc[3][4 * f4 + 1]);
+        acc[3][4 * f4 + 2] = fmaf(x.w, w.z, acc[3][4 * f4 + 2]);
+        acc[3][4 * f4 + 3] = fmaf(x.w, w.w, acc[3][4 * f4 + 3]);
+      }
+    }
+    __syncthreads();                 // the buffer is refilled two chunks later
+  }
+  // hidden activation and output projection; partial sums of the 16 hidden groups
+  const float* b1 = a.st.b1 + (size_t)h * dm.Fp + tn * NH;
+  const float* w2 = a.st.w2 + (size_t)h * dm.Fp + tn * NH;
+  float* red = Wc;                                                 // [16][UT2]
+  float part[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int f = 0; f < NH; ++f) {
+    const float bb = b1[f], ww = w2[f];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) part[r] = fmaf(ww, scorer_act(acc[r][f] + bb, dm.act), part[r]);
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) red[tn * UT2 + tm * 4 + r] = part[r];
+  __syncthreads();
+  if (tid < nrow) {
+    float sum = 0.f;
+    for (int g = 0; g < 16; ++g) sum += red[g * UT2 + tid];
+    const int u = u0 + tid;
+    float* prio_out = a.prio + (size_t)lp * Pm;
+    prio_out[u] = static_priority(canon_score(sum + a.st.b2[h]), u, a.st.log_gamma, h);
   }
 }
 
@@ -334,13 +533,36 @@ __global__ void __launch_bounds__(NT2) prefill_select_kernel(SelectArgs<T> a) {
 
 size_t score_smem(const Dims& dm) { return ((size_t)3 * dm.d * UT + 32 * dm.d + UT * NT1) * 4; }
 
+// the register-tiled scorer serves F = 128 / 256 when its buffers fit
+int gemm_nh(const Dims& dm) {
+  if (dm.F != dm.Fp || !(dm.F == 128 || dm.F == 256)) return 0;
+  return dm.F / 16;
+}
+size_t gemm_smem(const Dims& dm) {
+  const size_t x = (size_t)3 * dm.d * XS2 * 4;
+  const size_t wbytes = (size_t)2 * KC2 * dm.F * 4;
+  const size_t stage = (size_t)(UT2 - 1 + dm.D) * dm.d * 4;
+  const size_t red = (size_t)16 * UT2 * 4;
+  return x + std::max(std::max(wbytes, stage), red);
+}
+bool gemm_ok(const Dims& dm) { return gemm_nh(dm) != 0 && gemm_smem(dm) <= 227 * 1024; }
+
 }  // namespace
 
 cudaError_t prepare_prefill(const Dims& dm) {
   const int smem = (int)score_smem(dm);
+  cudaError_t e;
   if (dm.dtype == KVPOP_F32)
-    return cudaFuncSetAttribute(prefill_score_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  return cudaFuncSetAttribute(prefill_score_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(prefill_score_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  else
+    e = cudaFuncSetAttribute(prefill_score_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess || !gemm_ok(dm)) return e;
+  const int gs = (int)gemm_smem(dm);
+  if (dm.dtype == KVPOP_F32)
+    return dm.F == 256 ? cudaFuncSetAttribute(prefill_score_gemm_kernel<float, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs)
+                       : cudaFuncSetAttribute(prefill_score_gemm_kernel<float, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs);
+  return dm.F == 256 ? cudaFuncSetAttribute(prefill_score_gemm_kernel<bf16, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs)
+                     : cudaFuncSetAttribute(prefill_score_gemm_kernel<bf16, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs);
 }
 
 template <typename T>
@@ -350,9 +572,15 @@ static cudaError_t prefill_t(const State& st, const Dims& dm, const void* Q, con
   const int pairs = n_seq * dm.H;
   ScoreArgs<T> sa{st, dm, (const T*)Q, (const T*)K, (const T*)V, plen,
                   override_ ? override_ : nullptr, prio, Pmax};
-  dim3 g1((Pmax + UT - 1) / UT, pairs);
   if (Pmax > 0) {
-    prefill_score_kernel<T><<<g1, NT1, override_ ? 0 : score_smem(dm), stream>>>(sa);
+    if (!override_ && gemm_ok(dm)) {
+      dim3 g2((Pmax + UT2 - 1) / UT2, pairs);
+      if (dm.F == 256) prefill_score_gemm_kernel<T, 16><<<g2, NT3, gemm_smem(dm), stream>>>(sa);
+      else prefill_score_gemm_kernel<T, 8><<<g2, NT3, gemm_smem(dm), stream>>>(sa);
+    } else {
+      dim3 g1((Pmax + UT - 1) / UT, pairs);
+      prefill_score_kernel<T><<<g1, NT1, override_ ? 0 : score_smem(dm), stream>>>(sa);
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

@@ -268,3 +268,31 @@ def test_misaligned_and_bad_arguments(cuda_device):
     assert ei.value.status == 1
     c.check()
     c.free()
+
+
+@pytest.mark.parametrize("F,act,kv_only", [(256, "gelu", False), (128, "gelu", False),
+                                           (256, "silu", True)])
+def test_prefill_scores_against_oracle(cuda_device, F, act, kv_only):
+    """Prompt scorer (register-tiled for F = 128 / 256): stored priorities of the kept
+    slots equal the oracle's fp32 scores within 2e-5 relative, and the kept sets agree."""
+    cfg = get_config("q4b", batch=2, prompt_len=700, budget_B=200, scorer_hidden=F,
+                     scorer_act=act, scorer_kv_only=kv_only, log_gamma=-1e-3)
+    w = gen.scorer_weights(cfg)
+    L = [700, 437]
+    cache = make_cache(cfg, w)
+    gpu_prefill(cache, cfg, L, cuda_device)
+    pairs = all_pairs(cfg)
+    pre = oracle_pairs(cfg, w, L, 0, pairs)
+    agree = []
+    for (b, h), tr in zip(pairs, pre):
+        pos, sc = cache.pair_state(b, h)
+        o = set(tr.cache.kept_positions())
+        agree.append(len(o & set(pos)) / max(1, len(o)))
+        prio = {int(p): float(v) for p, v in zip(tr.cache.slot_pos[:tr.cache.n_valid],
+                                                  tr.cache.slot_prio[:tr.cache.n_valid])}
+        for p_, s_ in zip(pos, sc):
+            if p_ in prio:
+                assert abs(s_ - prio[p_]) <= 2e-5 * (1.0 + abs(prio[p_])), (b, h, p_)
+    print(f"prefill scorer F={F} {act} kv_only={kv_only}: kept-set agreement {np.mean(agree):.4f}")
+    assert np.mean(agree) >= 0.99
+    cache.free()
