@@ -112,12 +112,14 @@ def measured_peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
-def committed_traffic(config_name: str):
-    """DRAM bytes per attention launch from the committed ncu summary, if it matches the source."""
-    if not os.path.exists(TRAFFIC_FILE):
+def committed_traffic(config_name: str, path: str = TRAFFIC_FILE, sequences: int = 0):
+    """DRAM bytes per launch from a committed ncu summary, if it matches the source.
+
+    With ``sequences`` the captured figure is scaled from the capture's sequence count."""
+    if not os.path.exists(path):
         return None
     kv = {}
-    with open(TRAFFIC_FILE) as f:
+    with open(path) as f:
         for line in f:
             parts = line.split()
             if len(parts) >= 2 and not line.startswith("#"):
@@ -130,8 +132,11 @@ def committed_traffic(config_name: str):
     if kv.get("source_sha256") != sha or kv.get("config") != config_name:
         return None
     try:
-        return int(float(kv["dram_bytes_per_launch"]))
-    except (KeyError, ValueError):
+        v = float(kv["dram_bytes_per_launch"])
+        if sequences:
+            v *= sequences / float(kv["capture_sequences"])
+        return int(v)
+    except (KeyError, ValueError, ZeroDivisionError):
         return None
 
 
@@ -799,6 +804,10 @@ def run_prompt_bench(args):
         stream.synchronize()
     e2e_s = (time.perf_counter() - t0) / E
     tokens = n * P * world
+    tfile = os.path.join(ROOT, "profiles", ("prompt_t5_kernel_traffic.txt" if args.workload == "prompt"
+                                            else "target_t5_kernel_traffic.txt"))
+    traffic = (committed_traffic(cfg.name, tfile, sequences=n)
+               if (cfg.kv_dtype == "bf16" and d == 128 and not over) else None)
     if args.workload == "prompt":
         metric = "prompt tokens/sec with outputs under the running top-k mask (1 GB300)"
         kname = "prompt_tc_kernel" if cfg.kv_dtype == "bf16" else "prompt_simt_kernel"
@@ -821,7 +830,7 @@ def run_prompt_bench(args):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "roofline": {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak,
                      "peak_source": peak_src, "unit": "TFLOP/s", "frac": achieved / peak,
-                     "traffic": None, "algorithmic_flops_per_launch": flops, "ms_per_launch": k_ms},
+                     "traffic": traffic, "algorithmic_flops_per_launch": flops, "ms_per_launch": k_ms},
         "e2e": {"value": tokens / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": E,
                 "how": "pinned host inputs copied in, outputs copied out, inside the timed region"},
