@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkvpop.so")
 SOURCES = ["kvpop_api.cu", "kvpop_ingest.cu", "kvpop_ingest_cluster.cu", "kvpop_attend.cu", "kvpop_attend_tc.cu",
-           "kvpop_prefill.cu", "kvpop_noalloc.cu", "kvpop_mlstm.cu", "kvpop_topk.cu", "kvpop_prompt.cu", "kvpop_prompt_tc5.cu", "kvpop_target.cu"]
+           "kvpop_prefill.cu", "kvpop_noalloc.cu", "kvpop_mlstm.cu", "kvpop_topk.cu", "kvpop_prompt.cu", "kvpop_prompt_tc5.cu", "kvpop_target.cu",
+           "kvpop_score_tf32.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -1,6 +1,7 @@
 // Host side of the C ABI declared in include/kvpop.h: argument checks, device
 // memory, kernel launches.  No call throws or aborts; every failure is a status.
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -30,6 +31,9 @@ struct kvpop_cache {
   float* W1s = nullptr;                 // slice-major scorer weights for it
   float* b1s = nullptr;
   float* w2s = nullptr;
+  float* w1t = nullptr;                 // W1^T split for the tensor-core prompt scorer
+  std::vector<unsigned char> sc_maps;   // its TMA descriptors
+  bool use_tf32 = false;
   bool mlstm = false;                   // stateful mLSTM scorer instead of the MLP
   MlstmDev md{};
   // staging for kvpop_decode_step_host
@@ -96,6 +100,11 @@ void release(kvpop_cache* c) {
 // 64-byte aligned view of the stored TMA descriptors.
 void* tc_map_ptr(kvpop_cache* c) {
   uintptr_t p = reinterpret_cast<uintptr_t>(c->tc_maps.data());
+  return reinterpret_cast<void*>((p + 63) & ~uintptr_t(63));
+}
+void* sc_map_ptr(kvpop_cache* c) {
+  if (!c->use_tf32) return nullptr;
+  uintptr_t p = reinterpret_cast<uintptr_t>(c->sc_maps.data());
   return reinterpret_cast<void*>((p + 63) & ~uintptr_t(63));
 }
 
@@ -299,6 +308,12 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest_cluster(dm)));
   }
   if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_prefill(dm)));
+  c->use_tf32 = !c->mlstm && score_tf32_ok(dm) && std::getenv("KVPOP_PROMPT_SCORER_SIMT") == nullptr;
+  if (s == KVPOP_OK && c->use_tf32) {
+    s = dev_alloc(c, &p, 2 * H * dm.F * I * 4);
+    c->w1t = (float*)p;
+    c->sc_maps.assign(score_tf32_maps_size() + 64, 0);
+  }
   if (s == KVPOP_OK) {
     float* W1 = w;
     float* b1 = W1 + H * I * Fp;
@@ -317,6 +332,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     if (e == cudaSuccess && sc)
       e = NOTE(cudaMemcpy2DAsync(w2, Fp * 4, sc->w2, F * 4, F * 4, H, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && sc) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
+    if (e == cudaSuccess && c->use_tf32) e = NOTE(prepare_score_tf32(dm, W1, c->w1t, sc_map_ptr(c), stream));
     std::vector<float> minus_inf;
     if (c->mlstm) {
       // mLSTM weights: column blocks of Wcat [2d][NC] = [W_k | W_v | W_q | w_i | w_f | 0]
@@ -484,7 +500,8 @@ kvpop_status prefill_impl(kvpop_cache* c, const void* Q, const void* K, const vo
       e = NOTE(launch_prefill_select(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, prio,
                                      stream));
   } else if (e == cudaSuccess) {
-    e = NOTE(launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio, stream));
+    e = NOTE(launch_prefill(c->st, c->dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, prio,
+                            sc_map_ptr(c), stream));
   }
   if (e == cudaSuccess && outputs && Pmax > 0) {
     int32_t* rank = rank_out ? rank_out : reinterpret_cast<int32_t*>(base + rank_off);

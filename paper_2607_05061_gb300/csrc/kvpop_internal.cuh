@@ -118,10 +118,22 @@ cudaError_t tc_config(const Dims& dm, AttendConfig* out);
 cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const void* q, float* out,
                       int grid, cudaStream_t stream);
 
+// Prefill scores + selection; `tf32_maps` (W1^T tensor maps from prepare_score_tf32, or
+// null) routes the learned scores through the tensor-core scorer.
 cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const void* K,
                            const void* V, const int32_t* plen_dev, int first_seq, int n_seq,
                            int Pmax, const float* override_, float* tmp_prio,
-                           cudaStream_t stream);
+                           const void* tf32_maps, cudaStream_t stream);
+// Prompt scorer on the tensor cores (3xTF32 split products, fp32 accuracy): W1^T
+// split into tf32 head and residual [2][H][F][3d] (w1t, 2 H F 3d floats) and two
+// TMA descriptors over them (score_tf32_maps_size bytes, 64-byte aligned).
+bool score_tf32_ok(const Dims& dm);
+size_t score_tf32_maps_size();
+cudaError_t prepare_score_tf32(const Dims& dm, const float* W1, float* w1t, void* maps_out,
+                               cudaStream_t stream);
+cudaError_t launch_score_tf32(const State& st, const Dims& dm, const void* maps, const void* Q,
+                              const void* K, const void* V, const int32_t* plen, int n_seq, int Pmax,
+                              float* prio, cudaStream_t stream);
 
 // Running top-k over a prompt (App. C): static ranks and per-query cutoffs of
 // n_rows rows of S tokens; row r has len[r / rows_per_len] tokens (S if len is

@@ -568,12 +568,16 @@ cudaError_t prepare_prefill(const Dims& dm) {
 template <typename T>
 static cudaError_t prefill_t(const State& st, const Dims& dm, const void* Q, const void* K,
                              const void* V, const int32_t* plen, int first_seq, int n_seq,
-                             int Pmax, const float* override_, float* prio, cudaStream_t stream) {
+                             int Pmax, const float* override_, float* prio, const void* tf32_maps,
+                             cudaStream_t stream) {
   const int pairs = n_seq * dm.H;
   ScoreArgs<T> sa{st, dm, (const T*)Q, (const T*)K, (const T*)V, plen,
                   override_ ? override_ : nullptr, prio, Pmax};
   if (Pmax > 0) {
-    if (!override_ && gemm_ok(dm)) {
+    if (!override_ && tf32_maps) {
+      cudaError_t e = launch_score_tf32(st, dm, tf32_maps, Q, K, V, plen, n_seq, Pmax, prio, stream);
+      if (e != cudaSuccess) return e;
+    } else if (!override_ && gemm_ok(dm)) {
       dim3 g2((Pmax + UT2 - 1) / UT2, pairs);
       if (dm.F == 256) prefill_score_gemm_kernel<T, 16><<<g2, NT3, gemm_smem(dm), stream>>>(sa);
       else prefill_score_gemm_kernel<T, 8><<<g2, NT3, gemm_smem(dm), stream>>>(sa);
@@ -608,10 +612,12 @@ cudaError_t launch_prefill_select(const State& st, const Dims& dm, const void* Q
 cudaError_t launch_prefill(const State& st, const Dims& dm, const void* Q, const void* K,
                            const void* V, const int32_t* plen_dev, int first_seq, int n_seq,
                            int Pmax, const float* override_, float* tmp_prio,
-                           cudaStream_t stream) {
+                           const void* tf32_maps, cudaStream_t stream) {
   if (dm.dtype == KVPOP_F32)
-    return prefill_t<float>(st, dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, tmp_prio, stream);
-  return prefill_t<bf16>(st, dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, tmp_prio, stream);
+    return prefill_t<float>(st, dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, tmp_prio,
+                            tf32_maps, stream);
+  return prefill_t<bf16>(st, dm, Q, K, V, plen_dev, first_seq, n_seq, Pmax, override_, tmp_prio,
+                         tf32_maps, stream);
 }
 
 }  // namespace kvpop

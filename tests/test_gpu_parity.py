@@ -273,8 +273,9 @@ def test_misaligned_and_bad_arguments(cuda_device):
 @pytest.mark.parametrize("F,act,kv_only", [(256, "gelu", False), (128, "gelu", False),
                                            (256, "silu", True)])
 def test_prefill_scores_against_oracle(cuda_device, F, act, kv_only):
-    """Prompt scorer (register-tiled for F = 128 / 256): stored priorities of the kept
-    slots equal the oracle's fp32 scores within 2e-5 relative, and the kept sets agree."""
+    """Prompt scorer (3xTF32 tensor-core GEMM for F = 128 / 256): stored priorities of
+    the kept slots equal the oracle's fp32 scores within 2e-5 relative, and the kept
+    sets agree."""
     cfg = get_config("q4b", batch=2, prompt_len=700, budget_B=200, scorer_hidden=F,
                      scorer_act=act, scorer_kv_only=kv_only, log_gamma=-1e-3)
     w = gen.scorer_weights(cfg)
