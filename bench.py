@@ -810,12 +810,14 @@ def run_prompt_bench(args):
                if (cfg.kv_dtype == "bf16" and d == 128 and not over) else None)
     if args.workload == "prompt":
         metric = "prompt tokens/sec with outputs under the running top-k mask (1 GB300)"
-        kname = "prompt_tc_kernel" if cfg.kv_dtype == "bf16" else "prompt_simt_kernel"
+        kname = (("prompt_t5_kernel" if d == 128 and not os.environ.get("KVPOP_PROMPT_MMA_SYNC")
+                  else "prompt_tc_kernel") if cfg.kv_dtype == "bf16" else "prompt_simt_kernel")
         what = ("kvpop_prefill_attend: delayed scorer on every prompt token, prompt compression, "
                 "static ranks + running top-k cutoffs, masked causal attention with y and LSE")
     else:
         metric = "future-target tokens/sec (transposed attention pass + aggregation, 1 GB300)"
-        kname = "target_tc_kernel" if cfg.kv_dtype == "bf16" else "target_simt_kernel"
+        kname = (("target_t5_kernel" if d == 128 and not os.environ.get("KVPOP_TARGET_MMA_SYNC")
+                  else "target_tc_kernel") if cfg.kv_dtype == "bf16" else "target_simt_kernel")
         what = ("kvpop_future_target with the prompt pass's sparse LSE: log future mass per key "
                 "and query head, max aggregation, count normalisation")
     rec = {

@@ -23,6 +23,8 @@
 // Every wait is bounded; an expired wait records an error code and stops the CTA.
 #include <cuda.h>
 
+#include <type_traits>
+
 #include "kvpop_internal.cuh"
 #include "kvpop_ptx.cuh"
 #include "kvpop_tc05.cuh"
@@ -85,6 +87,13 @@ __device__ __forceinline__ bool builders_and(bool v) {
   return r != 0;
 }
 
+// Input dims [dim, dim + 32) of x_u = [k; v; qbar] handled at step c: the steps run
+// qbar, k, v chunks in turn so that the k / v loads of a step are issued during the one before.
+__host__ __device__ inline int chunk_dim(int c, int d) {
+  const int i = c / 3, r = c - 3 * i;
+  return (r == 0 ? 2 * d : r == 1 ? 0 : d) + i * SC_KC;
+}
+
 struct ScOff {
   int w, qm, b1, w2, red, bar, tmem, total;
 };
@@ -101,14 +110,14 @@ __host__ __device__ inline ScOff sc_offsets(int F, int D) {
   return o;
 }
 
-template <typename T, int F>
+template <typename T, int F, int G>
 __global__ void __launch_bounds__(SC_THREADS, 1)
     score_tf32_kernel(const __grid_constant__ CUtensorMap mhi, const __grid_constant__ CUtensorMap mlo,
                       ScArgs a) {
   extern __shared__ __align__(1024) unsigned char smf[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int lp = blockIdx.y, H = a.H, bl = lp / H, h = lp - bl * H;
-  const int d = a.d, D = a.D, G = a.G;
+  const int d = a.d, D = a.D;
   const int P = a.plen[bl];
   const int n_elig = max(P - D, 0);
   const int u0 = blockIdx.x * SC_M;
@@ -150,8 +159,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
       constexpr uint32_t WB = F * SC_KC * 4;
       auto tma_w = [&](int c, int b) {
         mbar_arrive_expect_tx(bar(2 + b), 2 * WB);
-        tma_2d(sb + off.w + (2 * b + 0) * WB, &mhi, c * SC_KC, h * F, bar(2 + b));
-        tma_2d(sb + off.w + (2 * b + 1) * WB, &mlo, c * SC_KC, h * F, bar(2 + b));
+        tma_2d(sb + off.w + (2 * b + 0) * WB, &mhi, chunk_dim(c, d), h * F, bar(2 + b));
+        tma_2d(sb + off.w + (2 * b + 1) * WB, &mlo, chunk_dim(c, d), h * F, bar(2 + b));
       };
       int wpend[2] = {0, -1}, last = -1;     // W chunk in flight per buffer; last committed chunk
       tma_w(0, 0);
@@ -195,67 +204,76 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ builders
-    const int kv_chunks = d / SC_KC;                        // chunks per K (and per V)
-    bool ok = true;
+    using Raw = typename std::conditional<sizeof(T) == 4, float4, uint2>::type;   // 4 inputs
+    auto to4 = [](const Raw& u) -> float4 {
+      if constexpr (sizeof(T) == 4) {
+        return u;
+      } else {
+        const bf16* e = reinterpret_cast<const bf16*>(&u);
+        return make_float4(to_f(e[0]), to_f(e[1]), to_f(e[2]), to_f(e[3]));
+      }
+    };
+    auto ld = [](const T* p) -> Raw { return *reinterpret_cast<const Raw*>(p); };
     auto split_store = [&](uint32_t buf, int r, int g4, float4 v) {
       const float4 hi = make_float4(tf32_head(v.x), tf32_head(v.y), tf32_head(v.z), tf32_head(v.w));
       const float4 lo = make_float4(v.x - hi.x, v.y - hi.y, v.z - hi.z, v.w - hi.w);
       *reinterpret_cast<float4*>(smf + buf + tile_off(r, g4, SC_M)) = hi;
       *reinterpret_cast<float4*>(smf + buf + SC_XB + tile_off(r, g4, SC_M)) = lo;
     };
-    auto load4 = [&](const T* p) -> float4 {
-      if (sizeof(T) == 4) return *reinterpret_cast<const float4*>(p);
-      const uint2 u = *reinterpret_cast<const uint2*>(p);
-      const bf16* e = reinterpret_cast<const bf16*>(&u);
-      return make_float4(to_f(e[0]), to_f(e[1]), to_f(e[2]), to_f(e[3]));
+    constexpr int KVI = SC_M * (SC_KC / 4) / SC_BUILD;      // K/V items per thread per chunk
+    // raw K/V inputs of step c (k or v rows of the 128 tokens, 32 dims), zero past nrow
+    auto load_kv = [&](int c, Raw (&v)[KVI]) {
+      const int dim0 = chunk_dim(c, d);
+      const T* src = dim0 < d ? Kp + dim0 : Vp + (dim0 - d);
+#pragma unroll
+      for (int j = 0; j < KVI; ++j) {
+        const int it = tid + j * SC_BUILD, r = it >> 3, g4 = it & 7;
+        v[j] = r < nrow ? ld(src + (size_t)(u0 + r) * d + g4 * 4) : Raw{};
+      }
     };
+    Raw cur[KVI], nxt[KVI];
+    bool ok = true;
     for (int c = 0; c < nch; ++c) {
       const int b = c & 1;
+      const bool q_step = chunk_dim(c, d) >= 2 * d;
+      if (c + 1 < nch && chunk_dim(c + 1, d) < 2 * d) load_kv(c + 1, nxt);   // prefetch
       if (c >= 2) ok = mbar_wait(bar(4 + b), ((c - 2) >> 1) & 1, a.err, SCERR_WAIT);
       if (!builders_and(ok)) { ok = false; break; }
       const uint32_t buf = 2 * b * SC_XB;
-      if (c < 2 * kv_chunks) {
-        const T* src = c < kv_chunks ? Kp : Vp;
-        const int dim0 = (c % kv_chunks) * SC_KC;
-        float4 v[SC_M * (SC_KC / 4) / SC_BUILD];
+      if (!q_step) {
+        if (c == 0) load_kv(0, cur);
 #pragma unroll
-        for (int j = 0; j < SC_M * (SC_KC / 4) / SC_BUILD; ++j) {
-          const int it = tid + j * SC_BUILD, r = it >> 3, g4 = it & 7;
-          v[j] = r < nrow ? load4(src + (size_t)(u0 + r) * d + dim0 + g4 * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int j = 0; j < SC_M * (SC_KC / 4) / SC_BUILD; ++j) {
+        for (int j = 0; j < KVI; ++j) {
           const int it = tid + j * SC_BUILD;
-          split_store(buf, it >> 3, it & 7, v[j]);
+          split_store(buf, it >> 3, it & 7, to4(cur[j]));
         }
       } else {
-        const int dim0 = (c - 2 * kv_chunks) * SC_KC;
+        const int dim0 = chunk_dim(c, d) - 2 * d;
         const int npos = nrow - 1 + D;              // positions u0+1 .. u0+nrow-1+D
-        constexpr int QB = 4;                       // items per thread in flight
+        constexpr int QB = 4;                       // items per thread per pass (G QB loads in flight)
         for (int base = tid; base < npos * (SC_KC / 4); base += QB * SC_BUILD) {
-          float4 s4[QB];
+          Raw v[G][QB];
 #pragma unroll
-          for (int j = 0; j < QB; ++j) s4[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int g = 0; g < G; ++g) {
-            float4 v[QB];
+          for (int g = 0; g < G; ++g)
 #pragma unroll
             for (int j = 0; j < QB; ++j) {
               const int it = base + j * SC_BUILD, tt = it >> 3, g4 = it & 7;
-              v[j] = it < npos * (SC_KC / 4) ? load4(Qp + ((size_t)g * Pm + u0 + 1 + tt) * d + dim0 + g4 * 4)
-                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+              v[g][j] = it < npos * (SC_KC / 4) ? ld(Qp + ((size_t)g * Pm + u0 + 1 + tt) * d + dim0 + g4 * 4)
+                                                : Raw{};
             }
-#pragma unroll
-            for (int j = 0; j < QB; ++j) {
-              s4[j].x += v[j].x; s4[j].y += v[j].y; s4[j].z += v[j].z; s4[j].w += v[j].w;
-            }
-          }
           const float ig = 1.0f / (float)G;
 #pragma unroll
           for (int j = 0; j < QB; ++j) {
+            float4 s4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+              const float4 f = to4(v[g][j]);
+              s4.x += f.x; s4.y += f.y; s4.z += f.z; s4.w += f.w;
+            }
             const int it = base + j * SC_BUILD;
             if (it < npos * (SC_KC / 4))
               *reinterpret_cast<float4*>(qm + (it >> 3) * SC_KC + (it & 7) * 4) =
-                  make_float4(s4[j].x * ig, s4[j].y * ig, s4[j].z * ig, s4[j].w * ig);
+                  make_float4(s4.x * ig, s4.y * ig, s4.z * ig, s4.w * ig);
           }
         }
         asm volatile("bar.sync 1, %0;" ::"n"(SC_BUILD) : "memory");
@@ -274,6 +292,8 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
         }
         asm volatile("bar.sync 1, %0;" ::"n"(SC_BUILD) : "memory");   // staging reused next chunk
       }
+#pragma unroll
+      for (int j = 0; j < KVI; ++j) cur[j] = nxt[j];
       fence_async_smem();
       mbar_arrive(bar(b));
     }
@@ -330,21 +350,28 @@ typedef CUresult (*EncodeTiledFn2)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-template <typename T, int F>
-cudaError_t launch_f(const CUtensorMap* maps, const ScArgs& a, int n_pairs, cudaStream_t stream) {
+template <typename T, int F, int G>
+cudaError_t launch_g(const CUtensorMap* maps, const ScArgs& a, int n_pairs, cudaStream_t stream) {
   const ScOff off = sc_offsets(F, a.D);
-  auto k = score_tf32_kernel<T, F>;
+  auto k = score_tf32_kernel<T, F, G>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, off.total);
   if (e != cudaSuccess) return e;
   dim3 grid((a.Pmax + SC_M - 1) / SC_M, n_pairs);
   k<<<grid, SC_THREADS, off.total, stream>>>(maps[0], maps[1], a);
   return cudaGetLastError();
 }
+template <typename T, int F>
+cudaError_t launch_f(const CUtensorMap* maps, const ScArgs& a, int n_pairs, cudaStream_t stream) {
+  if (a.G == 4) return launch_g<T, F, 4>(maps, a, n_pairs, stream);
+  if (a.G == 2) return launch_g<T, F, 2>(maps, a, n_pairs, stream);
+  return launch_g<T, F, 1>(maps, a, n_pairs, stream);
+}
 
 }  // namespace
 
 bool score_tf32_ok(const Dims& dm) {
-  if (dm.F != dm.Fp || !(dm.F == 128 || dm.F == 256) || (3 * dm.d) % SC_KC != 0 || dm.d % SC_KC != 0)
+  if (dm.F != dm.Fp || !(dm.F == 128 || dm.F == 256) || dm.d % SC_KC != 0 ||
+      !(dm.G == 1 || dm.G == 2 || dm.G == 4))
     return false;
   return sc_offsets(dm.F, dm.D).total <= 227 * 1024;
 }

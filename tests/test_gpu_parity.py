@@ -270,14 +270,18 @@ def test_misaligned_and_bad_arguments(cuda_device):
     c.free()
 
 
-@pytest.mark.parametrize("F,act,kv_only", [(256, "gelu", False), (128, "gelu", False),
-                                           (256, "silu", True)])
-def test_prefill_scores_against_oracle(cuda_device, F, act, kv_only):
+@pytest.mark.parametrize("F,act,kv_only,G,dt,D", [(256, "gelu", False, 4, "bf16", 16),
+                                                 (128, "gelu", False, 4, "bf16", 16),
+                                                 (256, "silu", True, 4, "bf16", 16),
+                                                 (128, "identity", False, 2, "f32", 5),
+                                                 (256, "gelu", False, 1, "bf16", 33)])
+def test_prefill_scores_against_oracle(cuda_device, F, act, kv_only, G, dt, D):
     """Prompt scorer (3xTF32 tensor-core GEMM for F = 128 / 256): stored priorities of
     the kept slots equal the oracle's fp32 scores within 2e-5 relative, and the kept
     sets agree."""
     cfg = get_config("q4b", batch=2, prompt_len=700, budget_B=200, scorer_hidden=F,
-                     scorer_act=act, scorer_kv_only=kv_only, log_gamma=-1e-3)
+                     scorer_act=act, scorer_kv_only=kv_only, log_gamma=-1e-3, q_per_kv=G,
+                     kv_dtype=dt, delay_D=D)
     w = gen.scorer_weights(cfg)
     L = [700, 437]
     cache = make_cache(cfg, w)
@@ -294,6 +298,7 @@ def test_prefill_scores_against_oracle(cuda_device, F, act, kv_only):
         for p_, s_ in zip(pos, sc):
             if p_ in prio:
                 assert abs(s_ - prio[p_]) <= 2e-5 * (1.0 + abs(prio[p_])), (b, h, p_)
-    print(f"prefill scorer F={F} {act} kv_only={kv_only}: kept-set agreement {np.mean(agree):.4f}")
+    print(f"prefill scorer F={F} {act} kv_only={kv_only} G={G} {dt} D={D}: "
+          f"kept-set agreement {np.mean(agree):.4f}")
     assert np.mean(agree) >= 0.99
     cache.free()
