@@ -132,12 +132,19 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
         const int st = j % ST;
         if (j >= ST && !mbar_wait(bar(B_EMPTY + st), ((j / ST) - 1) & 1, a.err, T5ERR_WAIT)) break;
         const uint32_t kd = sb + OFF_KV + st * 2 * KVB, vd = kd + KVB;
-        for (int i = pt; i < T5_BN * 16; i += T5_PT) {
-          const int key = i >> 4, c = i & 15;
-          const int t = entry(j * T5_BN + key);
-          const uint32_t off = tile_off(key, c, T5_BN);
-          cp_async16(kd + off, Kp + (size_t)t * 128 + c * 8, 16);
-          if (WANT_Y) cp_async16(vd + off, Vp + (size_t)t * 128 + c * 8, 16);
+        // 8 threads per key row, 32 bytes (two 16-byte chunks) of K and of V each:
+        // one position lookup per row and thread, rows T5_PT / 8 apart
+        const int c2 = 2 * (pt & 7);
+#pragma unroll 2
+        for (int key = pt >> 3; key < T5_BN; key += T5_PT / 8) {
+          const size_t t = (size_t)entry(j * T5_BN + key) * 128 + c2 * 8;
+          const uint32_t o0 = tile_off(key, c2, T5_BN), o1 = tile_off(key, c2 + 1, T5_BN);
+          cp_async16(kd + o0, Kp + t, 16);
+          cp_async16(kd + o1, Kp + t + 8, 16);
+          if (WANT_Y) {
+            cp_async16(vd + o0, Vp + t, 16);
+            cp_async16(vd + o1, Vp + t + 8, 16);
+          }
         }
         cp_async_arrive_noinc(bar(B_FULL + st));
       }
