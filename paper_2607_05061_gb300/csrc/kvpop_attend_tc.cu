@@ -151,6 +151,9 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     }
     mbar_fence_init();
   }
+  // Launched as a programmatic dependent of the ingest: everything below reads the
+  // state it writes, so wait here for it to complete (a no-op without a predecessor).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   build_schedule<NT>(a.nvalid, a.len, npairs, a.D, TILE, prefix, scan);
   const long long Ttot = prefix[npairs];
   if (Ttot <= 0) return;
@@ -456,11 +459,21 @@ cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const v
   a.D = dm.D;
   a.ring_rows = tc_ring_rows(dm);
   a.qscale = kLog2e / sqrtf((float)dm.d);
+  // programmatic stream serialisation: the grid may be scheduled while the kernel
+  // before it (the ingest) finishes; the kernel waits for it before touching the state
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
 #define LAUNCH(HD_, G_)                                                                   \
   if (dm.d == HD_ && dm.G == G_) {                                                        \
-    attend_tc_kernel<HD_, G_><<<grid, TcTraits<HD_, G_>::THREADS, tc_smem<HD_, G_>(dm.pairs), \
-                                stream>>>(m->sk, m->sv, m->rk, m->rv, a);                 \
-    return cudaGetLastError();                                                            \
+    cfg.blockDim = dim3(TcTraits<HD_, G_>::THREADS, 1, 1);                                \
+    cfg.dynamicSmemBytes = tc_smem<HD_, G_>(dm.pairs);                                    \
+    return cudaLaunchKernelEx(&cfg, attend_tc_kernel<HD_, G_>, m->sk, m->sv, m->rk, m->rv, a); \
   }
   TC_CASES(LAUNCH)
 #undef LAUNCH

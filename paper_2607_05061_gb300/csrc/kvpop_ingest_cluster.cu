@@ -115,6 +115,9 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
   // sequences of this cluster: group*SBC + j; CTA `rank` owns j = OWN*rank + o
   const int own_b0 = group * SBC + OWN * (int)rank;
 
+  // the attention that follows may be scheduled now; it waits for this grid to complete
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
   // ---- issue every load this CTA needs ------------------------------------------------
   if (tid == 0) {
     mbar_init(smem_u32(&bar), 1);
@@ -265,23 +268,46 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
   cluster_sync();   // every X row is in every CTA
 
   // ---- this CTA's hidden slice for all 16 sequences --------------------------------------
+  // Thread (f, ks) accumulates hidden unit f over input slice ks for every sequence: per
+  // 4 inputs, 4 weights and 16 broadcast input vectors feed 64 FMAs.  The slices' partial
+  // sums meet in shared memory (over the input rows, no longer needed), then warp w adds
+  // b1, applies the activation and contracts with w2 for sequences 2w, 2w+1.
   {
-    const int j0 = 2 * warp, j1 = 2 * warp + 1;
-    const float* x0 = X + (size_t)j0 * in_dim;
-    const float* x1 = X + (size_t)j1 * in_dim;
-    float c0 = 0.f, c1 = 0.f;
-    for (int f = lane; f < FS; f += 32) {
-      float a0 = b1s[f], a1 = a0;
-#pragma unroll 4
-      for (int i = 0; i < in_dim; i += 4) {
-        const float4 u0 = *reinterpret_cast<const float4*>(x0 + i);
-        const float4 u1 = *reinterpret_cast<const float4*>(x1 + i);
+    // input slices (FS <= 64); NKS * FS <= 3d keeps the partial sums inside the input rows
+    const int NKS = min(NT / FS, in_dim / FS);
+    const int SL = ((in_dim + NKS - 1) / NKS + 3) & ~3;   // inputs per slice, multiple of 4
+    const int f = tid % FS, ks = tid / FS;
+    float acc[SBC];
+#pragma unroll
+    for (int j = 0; j < SBC; ++j) acc[j] = 0.f;
+    if (ks < NKS) {
+      const int i_end = min(in_dim, (ks + 1) * SL);
+      for (int i = ks * SL; i < i_end; i += 4) {
         const float w0 = Ws[(i + 0) * FS + f], w1 = Ws[(i + 1) * FS + f];
         const float w2 = Ws[(i + 2) * FS + f], w3 = Ws[(i + 3) * FS + f];
-        a0 = fmaf(u0.x, w0, a0); a0 = fmaf(u0.y, w1, a0); a0 = fmaf(u0.z, w2, a0); a0 = fmaf(u0.w, w3, a0);
-        a1 = fmaf(u1.x, w0, a1); a1 = fmaf(u1.y, w1, a1); a1 = fmaf(u1.z, w2, a1); a1 = fmaf(u1.w, w3, a1);
+#pragma unroll
+        for (int j = 0; j < SBC; ++j) {
+          const float4 u = *reinterpret_cast<const float4*>(X + (size_t)j * in_dim + i);
+          acc[j] = fmaf(u.x, w0, fmaf(u.y, w1, fmaf(u.z, w2, fmaf(u.w, w3, acc[j]))));
+        }
       }
-      const float wf = w2s[f];
+    }
+    __syncthreads();                                  // every thread is done with X
+    float* red = X;                                   // [NKS][SBC][FS] partial sums
+    if (ks < NKS) {
+#pragma unroll
+      for (int j = 0; j < SBC; ++j) red[((size_t)ks * SBC + j) * FS + f] = acc[j];
+    }
+    __syncthreads();
+    float c0 = 0.f, c1 = 0.f;
+    const int j0 = 2 * warp, j1 = 2 * warp + 1;
+    for (int ff = lane; ff < FS; ff += 32) {
+      float a0 = b1s[ff], a1 = a0;
+      for (int kk = 0; kk < NKS; ++kk) {
+        a0 += red[((size_t)kk * SBC + j0) * FS + ff];
+        a1 += red[((size_t)kk * SBC + j1) * FS + ff];
+      }
+      const float wf = w2s[ff];
       c0 = fmaf(wf, scorer_act(a0, dm.act), c0);
       c1 = fmaf(wf, scorer_act(a1, dm.act), c1);
     }
