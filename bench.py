@@ -735,20 +735,21 @@ def run_prompt_bench(args):
     lse = torch.empty((n, H * G, P), dtype=torch.float32, device=dev)
     rk = torch.empty((n, H, P), dtype=torch.int32, device=dev)
     tu = torch.empty((n, H, P), dtype=torch.int32, device=dev)
+    od = torch.empty((n, H, P), dtype=torch.int32, device=dev)
     logm = torch.empty((n, H * G, P), dtype=torch.float32, device=dev)
     tgt = torch.empty((n, H, P), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     k_b = cfg.budget_B - cfg.n_sink
 
     def prompt_step():
-        cache.prefill_attend(Q, K, V, L, Y, lse, rank=rk, tau=tu)
+        cache.prefill_attend(Q, K, V, L, Y, lse, rank=rk, tau=tu, order=od)
 
     def target_step():
         kvpop.future_target(Q, K, lse, cfg.delay_D, logm=logm, target=tgt)
 
     def kernel_only():
         if args.workload == "prompt":
-            kvpop.prompt_attention(Q, K, V, rk, tu, cfg.n_sink, cfg.delay_D, k_b, Y=Y, lse=lse)
+            kvpop.prompt_attention(Q, K, V, rk, tu, cfg.n_sink, cfg.delay_D, k_b, Y=Y, lse=lse, order=od)
         else:
             kvpop.future_target(Q, K, lse, cfg.delay_D, logm=logm, want_target=False)
 

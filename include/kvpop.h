@@ -161,6 +161,9 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* cache, const void* Q_dev, const
  *            normaliser over the retained keys (the sparse LSE of App. D.3),
  *            or NULL
  *   rank_dev, tau_dev [n_seq][H][Pmax] int32 out (-1 past P), or NULL
+ *   order_dev [n_seq][H][Pmax] int32 out, position of each rank (entries from P on
+ *            untouched), or NULL; with rank_dev and tau_dev it is what
+ *            kvpop_prompt_attention takes to recompute the outputs
  * Other arguments as kvpop_prefill_compress.  Needs Pmax <= 262144,
  * n_seq*H <= 65535, d in {64, 128}, G in {1, 2, 4} and per-tile key lists of
  * 4*(B + s + 2*128 + D) bytes that fit in shared memory (else
@@ -170,7 +173,8 @@ kvpop_status kvpop_prefill_attend(kvpop_cache* cache, const void* Q_dev, const v
                                   const void* V_dev, const int32_t* prompt_len_host,
                                   int32_t first_seq, int32_t n_seq, int32_t Pmax,
                                   const float* score_override_dev, float* Y_dev, float* lse_dev,
-                                  int32_t* rank_dev, int32_t* tau_dev, cudaStream_t stream);
+                                  int32_t* rank_dev, int32_t* tau_dev, int32_t* order_dev,
+                                  cudaStream_t stream);
 
 /* Bytes of device workspace kvpop_topk_cutoff needs (0 for an empty problem). */
 size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S);
@@ -184,6 +188,8 @@ size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S);
  *   tau_dev  [n_rows][S]  rank of the min(k, |E(q)|)-th best token of
  *                         E(q) = {n_sink <= t <= q - window}; -1 while E(q) is
  *                         empty and past the row length
+ *   order_dev [n_rows][S] (or NULL) position of each rank: order[r][rank[r][t]] = t
+ *                         for t below the row length (entries past it untouched)
  * Where Algorithm 2 leaves tau_q = -1 while fewer than k tokens are eligible,
  * this keeps all of them (the top k of a set smaller than k is the set).
  * workspace_dev: kvpop_topk_workspace_bytes(n_rows, S) bytes, 256-byte aligned,
@@ -191,8 +197,8 @@ size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S);
  * `stream`; no allocation. */
 kvpop_status kvpop_topk_cutoff(const float* prio_dev, const int32_t* lengths_dev, int32_t n_rows,
                                int32_t S, int32_t n_sink, int32_t window, int32_t k,
-                               int32_t* rank_dev, int32_t* tau_dev, void* workspace_dev,
-                               size_t workspace_bytes, cudaStream_t stream);
+                               int32_t* rank_dev, int32_t* tau_dev, int32_t* order_dev,
+                               void* workspace_dev, size_t workspace_bytes, cudaStream_t stream);
 
 /* Masked causal attention over prompts under the running top-k mask given by
  * rank / tau from kvpop_topk_cutoff (same n_sink, window and k), no cache
@@ -200,13 +206,17 @@ kvpop_status kvpop_topk_cutoff(const float* prio_dev, const int32_t* lengths_dev
  *   y[q] = sum_t softmax_t(M[q,t] ? q.k_t / sqrt(d) : -inf) v_t
  *   Q_dev [n_seq][H*G][S][d], K_dev, V_dev [n_seq][H][S][d]  (dtype)
  *   rank_dev, tau_dev [n_seq][H][S] int32;  lengths_dev [n_seq] or NULL (= S)
+ *   order_dev [n_seq][H][S] int32, the order output of the same kvpop_topk_cutoff
+ *   call, or NULL: with it a tile's key lists are built from the ranks up to its
+ *   largest cutoff when that is shorter than its eligible positions (same outputs)
  *   Y_dev [n_seq][H*G][S][d] fp32 out; lse_dev [n_seq][H*G][S] fp32 out or NULL
  * Limits as kvpop_prefill_attend.  Asynchronous on `stream`; no allocation.
  * rank / tau that did not come from kvpop_topk_cutoff give unspecified outputs
  * but never an out-of-bounds access. */
 kvpop_status kvpop_prompt_attention(const void* Q_dev, const void* K_dev, const void* V_dev,
                                     const int32_t* rank_dev, const int32_t* tau_dev,
-                                    const int32_t* lengths_dev, int32_t n_seq, int32_t n_kv_heads,
+                                    const int32_t* order_dev, const int32_t* lengths_dev,
+                                    int32_t n_seq, int32_t n_kv_heads,
                                     int32_t q_per_kv, int32_t head_dim, int32_t S, int32_t n_sink,
                                     int32_t window, int32_t k, kvpop_dtype dtype, float* Y_dev,
                                     float* lse_dev, cudaStream_t stream);

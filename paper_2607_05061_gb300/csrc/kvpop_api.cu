@@ -450,7 +450,7 @@ namespace {
 kvpop_status prefill_impl(kvpop_cache* c, const void* Q, const void* K, const void* V,
                           const int32_t* plen_host, int32_t first_seq, int32_t n_seq, int32_t Pmax,
                           const float* override_, float* Y, float* lse, int32_t* rank_out,
-                          int32_t* tau_out, cudaStream_t stream) {
+                          int32_t* tau_out, int32_t* order_out, cudaStream_t stream) {
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
   if (!plen_host || n_seq < 0 || first_seq < 0 || first_seq + (long long)n_seq > c->dm.batch ||
@@ -508,10 +508,12 @@ kvpop_status prefill_impl(kvpop_cache* c, const void* Q, const void* K, const vo
     int32_t* tau = tau_out ? tau_out : reinterpret_cast<int32_t*>(base + tau_off);
     const int s_ = c->dm.s, D = c->dm.D, k = c->dm.B - c->dm.s;
     e = NOTE(launch_topk(prio, plen_dev, c->dm.H, D, (int)pairs, Pmax, s_, D, k, rank, tau,
-                         base + ws_off, stream));
+                         order_out, base + ws_off, stream));
+    const int32_t* order = order_out ? order_out : topk_order(base + ws_off, (int)pairs, Pmax);
     if (e == cudaSuccess)
-      e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, plen_dev, n_seq, c->dm.H, c->dm.G, c->dm.d,
-                                    Pmax, s_, D, k, c->dm.dtype, Y, lse, c->st.err, stream));
+      e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, order,
+                                    plen_dev, n_seq, c->dm.H, c->dm.G, c->dm.d, Pmax, s_, D, k,
+                                    c->dm.dtype, Y, lse, c->st.err, stream));
   }
   // the host copy of the lengths must outlive the async copy
   if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
@@ -526,16 +528,18 @@ kvpop_status kvpop_prefill_compress(kvpop_cache* c, const void* Q, const void* K
                                     const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
                                     int32_t Pmax, const float* override_, cudaStream_t stream) {
   return prefill_impl(c, Q, K, V, plen_host, first_seq, n_seq, Pmax, override_, nullptr, nullptr,
-                      nullptr, nullptr, stream);
+                      nullptr, nullptr, nullptr, stream);
 }
 
 kvpop_status kvpop_prefill_attend(kvpop_cache* c, const void* Q, const void* K, const void* V,
                                   const int32_t* plen_host, int32_t first_seq, int32_t n_seq,
                                   int32_t Pmax, const float* override_, float* Y, float* lse,
-                                  int32_t* rank_out, int32_t* tau_out, cudaStream_t stream) {
+                                  int32_t* rank_out, int32_t* tau_out, int32_t* order_out,
+                                  cudaStream_t stream) {
   if (!Y) return KVPOP_ERR_INVALID_ARG;
+  if (!aligned4(order_out)) return KVPOP_ERR_ALIGN;
   return prefill_impl(c, Q, K, V, plen_host, first_seq, n_seq, Pmax, override_, Y, lse, rank_out,
-                      tau_out, stream);
+                      tau_out, order_out, stream);
 }
 
 size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S) {
@@ -545,22 +549,24 @@ size_t kvpop_topk_workspace_bytes(int32_t n_rows, int32_t S) {
 
 kvpop_status kvpop_topk_cutoff(const float* prio, const int32_t* lengths, int32_t n_rows, int32_t S,
                                int32_t n_sink, int32_t window, int32_t k, int32_t* rank, int32_t* tau,
-                               void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+                               int32_t* order, void* workspace, size_t workspace_bytes,
+                               cudaStream_t stream) {
   if (n_rows < 0 || S < 0 || S > kTopkMaxS || n_sink < 0 || window < 1 || k < 1)
     return KVPOP_ERR_INVALID_ARG;
   if (n_rows == 0 || S == 0) return KVPOP_OK;
   if (!prio || !rank || !tau || !workspace) return KVPOP_ERR_INVALID_ARG;
   if (workspace_bytes < topk_workspace_bytes(n_rows, S)) return KVPOP_ERR_INVALID_ARG;
   if (!aligned4(prio) || !aligned4(lengths) || !aligned4(rank) || !aligned4(tau) ||
-      (reinterpret_cast<uintptr_t>(workspace) & 255u))
+      !aligned4(order) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
     return KVPOP_ERR_ALIGN;
   cudaError_t e = NOTE(launch_topk(prio, lengths, 1, 0, n_rows, S, n_sink, window, k, rank, tau,
-                                   workspace, stream));
+                                   order, workspace, stream));
   return from_cuda(e);
 }
 
 kvpop_status kvpop_prompt_attention(const void* Q, const void* K, const void* V, const int32_t* rank,
-                                    const int32_t* tau, const int32_t* lengths, int32_t n_seq,
+                                    const int32_t* tau, const int32_t* order,
+                                    const int32_t* lengths, int32_t n_seq,
                                     int32_t n_kv_heads, int32_t q_per_kv, int32_t head_dim, int32_t S,
                                     int32_t n_sink, int32_t window, int32_t k, kvpop_dtype dtype,
                                     float* Y, float* lse, cudaStream_t stream) {
@@ -571,10 +577,10 @@ kvpop_status kvpop_prompt_attention(const void* Q, const void* K, const void* V,
   if (n_seq == 0 || S == 0) return KVPOP_OK;
   if (!Q || !K || !V || !rank || !tau || !Y) return KVPOP_ERR_INVALID_ARG;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(Y) || !aligned4(rank) ||
-      !aligned4(tau) || !aligned4(lengths) || !aligned4(lse))
+      !aligned4(tau) || !aligned4(order) || !aligned4(lengths) || !aligned4(lse))
     return KVPOP_ERR_ALIGN;
-  cudaError_t e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, lengths, n_seq, n_kv_heads, q_per_kv,
-                                            head_dim, S, n_sink, window, k, dtype, Y, lse,
+  cudaError_t e = NOTE(launch_prompt_attend(Q, K, V, rank, tau, order, lengths, n_seq, n_kv_heads,
+                                            q_per_kv, head_dim, S, n_sink, window, k, dtype, Y, lse,
                                             standalone_err(), stream));
   return from_cuda(e);
 }

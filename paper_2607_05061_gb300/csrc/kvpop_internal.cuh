@@ -140,15 +140,22 @@ cudaError_t launch_score_tf32(const State& st, const Dims& dm, const void* maps,
 // null), the last `tail` of them without a priority.
 constexpr int kTopkMaxS = 1 << 18;
 size_t topk_workspace_bytes(int n_rows, int S);
+// After launch_topk: the position of every rank of every row ([n_rows][S], ranks 0 .. L-1
+// of a row of length L), inside the workspace.
+const int32_t* topk_order(const void* workspace, int n_rows, int S);
+// `order` receives the position of each rank ([n_rows][S]); null puts it in the workspace
+// (topk_order).
 cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len, int tail,
                         int n_rows, int S, int s, int w, int k, int32_t* rank, int32_t* tau,
-                        void* workspace, cudaStream_t stream);
+                        int32_t* order, void* workspace, cudaStream_t stream);
 // Masked causal attention over a prompt under the running top-k mask.
 bool prompt_attend_ok(int dtype, int d, int G, int s, int w, int k);
+// `order` (positions by rank, from topk_order, or null) lets a tile's key lists be
+// built from the ranks up to its largest cutoff instead of from every eligible position.
 cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, const int32_t* rank,
-                                 const int32_t* tau, const int32_t* len, int n_seq, int H, int G,
-                                 int d, int S, int s, int w, int k, int dtype, float* Y, float* lse,
-                                 int32_t* err, cudaStream_t stream);
+                                 const int32_t* tau, const int32_t* order, const int32_t* len,
+                                 int n_seq, int H, int G, int d, int S, int s, int w, int k,
+                                 int dtype, float* Y, float* lse, int32_t* err, cudaStream_t stream);
 
 // Dense causal log-normalisers of every prompt query (LSE only, no output rows).
 cudaError_t launch_causal_lse(const void* Q, const void* K, const int32_t* len, int n_seq, int H,

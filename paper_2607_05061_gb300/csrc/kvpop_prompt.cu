@@ -454,11 +454,11 @@ bool prompt_attend_ok(int dtype, int d, int G, int s, int w, int k) {
 }
 
 cudaError_t launch_prompt_attend(const void* Q, const void* K, const void* V, const int32_t* rank,
-                                 const int32_t* tau, const int32_t* len, int n_seq, int H, int G,
-                                 int d, int S, int s, int w, int k, int dtype, float* Y, float* lse,
-                                 int32_t* err, cudaStream_t stream) {
+                                 const int32_t* tau, const int32_t* order, const int32_t* len,
+                                 int n_seq, int H, int G, int d, int S, int s, int w, int k,
+                                 int dtype, float* Y, float* lse, int32_t* err, cudaStream_t stream) {
   if (n_seq <= 0 || S <= 0) return cudaSuccess;
-  PromptArgs a{Q, K, V, rank, tau, len, Y, lse, H, G, S, s, w, s + k, 0,
+  PromptArgs a{Q, K, V, rank, tau, order, len, Y, lse, H, G, S, s, w, s + k, 0,
                1.4426950408889634f / sqrtf((float)d), err};
   return dispatch<false, true>(a, n_seq * H, dtype, d, G, stream);
 }
@@ -467,7 +467,7 @@ cudaError_t launch_causal_lse(const void* Q, const void* K, const int32_t* len, 
                               int G, int d, int S, int dtype, float* lse, int32_t* err,
                               cudaStream_t stream) {
   if (n_seq <= 0 || S <= 0) return cudaSuccess;
-  PromptArgs a{Q, K, nullptr, nullptr, nullptr, len, nullptr, lse, H, G, S, 0, 1, 0, 0,
+  PromptArgs a{Q, K, nullptr, nullptr, nullptr, nullptr, len, nullptr, lse, H, G, S, 0, 1, 0, 0,
                1.4426950408889634f / sqrtf((float)d), err};
   return dispatch<true, false>(a, n_seq * H, dtype, d, G, stream);
 }

@@ -17,6 +17,7 @@ struct PromptArgs {
   const void* V;
   const int32_t* rank;       // [n_seq*H][S]
   const int32_t* tau;        // [n_seq*H][S]
+  const int32_t* order;      // [n_seq*H][S] position of each rank, or nullptr
   const int32_t* len;        // [n_seq] or nullptr (= S)
   float* Y;                  // [n_seq][H*G][S][d]
   float* lse;                // [n_seq][H*G][S] or nullptr
@@ -84,22 +85,39 @@ __device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int
   for (int t = tid; t < nAs && t < a.capA; t += NT) posA[t] = t;
   for (int j = tid; j < nMs && j < a.capM; j += NT) posM[j] = nAs + j;
   int nA = nAs, nM = nMs;
-  // eligible for the whole tile: t in [s, q0 - w]
+  // eligible for the whole tile: t in [s, q0 - w].  The candidates are the eligible
+  // positions ranked within tmax: walk either the positions s .. hi (reading their ranks)
+  // or, when it is shorter, the ranks 0 .. tmax (reading their positions, kept if eligible).
   const int hi = q0 - w;
   constexpr int EPT = 16;
   if (hi >= s && tmax >= 0) {
-    for (int c0 = s; c0 <= hi; c0 += NT * EPT) {
-      const int t0 = c0 + tid * EPT;
-      int r[EPT];
+    const int32_t* order = a.order ? a.order + (size_t)ti.pair * a.S : nullptr;
+    const bool by_rank = order != nullptr && tmax < hi - s;
+    const int n_walk = by_rank ? tmax + 1 : hi - s + 1;
+    for (int c0 = 0; c0 < n_walk; c0 += NT * EPT) {
+      const int i0 = c0 + tid * EPT;
+      int r[EPT], t[EPT];
 #pragma unroll
-      for (int e = 0; e < EPT; ++e) r[e] = (t0 + e <= hi) ? __ldg(rank + t0 + e) : INT_MAX;
+      for (int e = 0; e < EPT; ++e) {
+        const int i = i0 + e;
+        if (i >= n_walk) {
+          r[e] = INT_MAX;
+          t[e] = 0;
+        } else if (by_rank) {
+          t[e] = __ldg(order + i);
+          r[e] = (t[e] >= s && t[e] <= hi) ? i : INT_MAX;
+        } else {
+          t[e] = s + i;
+          r[e] = __ldg(rank + s + i);
+        }
+      }
       int ca = 0, cm = 0;
 #pragma unroll
       for (int e = 0; e < EPT; ++e) {
         ca += r[e] <= tmin;
         cm += (r[e] > tmin) & (r[e] <= tmax);
       }
-      const int v = ca | (cm << 16);        // at most NT * EPT = 4096 per field
+      const int v = ca | (cm << 16);        // at most NT * EPT = 6144 per field
       int x = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -120,10 +138,10 @@ __device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int
 #pragma unroll
       for (int e = 0; e < EPT; ++e) {
         if (r[e] <= tmin) {
-          if (ia < a.capA) posA[ia] = t0 + e;
+          if (ia < a.capA) posA[ia] = t[e];
           ++ia;
         } else if (r[e] <= tmax) {
-          if (im < a.capM) posM[im] = t0 + e;
+          if (im < a.capM) posM[im] = t[e];
           ++im;
         }
       }

@@ -44,6 +44,7 @@ struct RankArgs {
   uint32_t* kb;
   int32_t* pb;
   int32_t* rank;             // [n_rows][S]
+  int32_t* order;            // [n_rows][S] position of each rank (inverse of rank; the pb buffer)
 };
 
 // Ascending key = descending priority; NaN -> -inf, -0 -> +0 (as the decode scores).
@@ -150,6 +151,7 @@ __global__ void __launch_bounds__(RK_NT) rank_kernel(RankArgs a) {
           dp[dst] = pos;
         } else {
           a.rank[ro + pos] = (int32_t)dst;
+          a.order[ro + dst] = pos;          // pb is free in the last pass
         }
       }
       __syncwarp();
@@ -284,9 +286,15 @@ size_t topk_workspace_bytes(int n_rows, int S) {
   return (size_t)n_rows * (size_t)S * 16 + 1024;
 }
 
+const int32_t* topk_order(const void* workspace, int n_rows, int S) {
+  const size_t n = (size_t)n_rows * S;
+  const size_t al = (n * 4 + 255) & ~size_t(255);
+  return reinterpret_cast<const int32_t*>(static_cast<const char*>(workspace) + 3 * al);
+}
+
 cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len, int tail,
                         int n_rows, int S, int s, int w, int k, int32_t* rank, int32_t* tau,
-                        void* workspace, cudaStream_t stream) {
+                        int32_t* order, void* workspace, cudaStream_t stream) {
   if (n_rows <= 0 || S <= 0) return cudaSuccess;
   const size_t n = (size_t)n_rows * S;
   char* ws = static_cast<char*>(workspace);
@@ -294,7 +302,8 @@ cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len,
   RankArgs ra{prio, len, rows_per_len, tail, n_rows, S,
               reinterpret_cast<uint32_t*>(ws), reinterpret_cast<int32_t*>(ws + al(n * 4)),
               reinterpret_cast<uint32_t*>(ws + 2 * al(n * 4)),
-              reinterpret_cast<int32_t*>(ws + 3 * al(n * 4)), rank};
+              reinterpret_cast<int32_t*>(ws + 3 * al(n * 4)), rank,
+              order ? order : reinterpret_cast<int32_t*>(ws + 3 * al(n * 4))};
   rank_kernel<<<n_rows, RK_NT, 0, stream>>>(ra);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;

@@ -69,11 +69,11 @@ _SIGS = {
     "kvpop_attend_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, c_int32, c_int32, c_int32,
                                             c_int32, c_int32, c_int32, ctypes.c_int, _P]),
     "kvpop_prefill_attend": (ctypes.c_int, [_P, _P, _P, _P, POINTER(c_int32), c_int32, c_int32,
-                                            c_int32, _P, _P, _P, _P, _P, _P]),
+                                            c_int32, _P, _P, _P, _P, _P, _P, _P]),
     "kvpop_topk_workspace_bytes": (c_size_t, [c_int32, c_int32]),
     "kvpop_topk_cutoff": (ctypes.c_int, [_P, _P, c_int32, c_int32, c_int32, c_int32, c_int32, _P, _P,
-                                         _P, c_size_t, _P]),
-    "kvpop_prompt_attention": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, c_int32, c_int32, c_int32,
+                                         _P, _P, c_size_t, _P]),
+    "kvpop_prompt_attention": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, c_int32, c_int32, c_int32,
                                               c_int32, c_int32, c_int32, c_int32, c_int32,
                                               ctypes.c_int, _P, _P, _P]),
     "kvpop_causal_lse": (ctypes.c_int, [_P, _P, _P, c_int32, c_int32, c_int32, c_int32, c_int32,
@@ -168,7 +168,7 @@ class KVpopCache:
                                    _ptr(override), _stream(stream)), "kvpop_prefill_compress")
 
     def prefill_attend(self, Q, K, V, prompt_lens: Sequence[int], Y, lse=None, first_seq: int = 0,
-                       override=None, rank=None, tau=None, stream=None):
+                       override=None, rank=None, tau=None, order=None, stream=None):
         """``prefill`` plus the prompt's outputs ``Y [n][H*G][Pmax][d]`` (fp32) under the
         running top-k mask; optionally the LSE, ranks and cutoffs."""
         n_seq = len(prompt_lens)
@@ -176,7 +176,7 @@ class KVpopCache:
         Pmax = K.shape[2]
         _ck(kvpop_prefill_attend(self.handle, _ptr(Q), _ptr(K), _ptr(V), arr, first_seq, n_seq, Pmax,
                                  _ptr(override), _ptr(Y), _ptr(lse), _ptr(rank), _ptr(tau),
-                                 _stream(stream)), "kvpop_prefill_attend")
+                                 _ptr(order), _stream(stream)), "kvpop_prefill_attend")
 
     def ingest(self, q, k, v, override=None, evict_info=None, score_out=None, stream=None):
         _ck(kvpop_decode_ingest(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(override),
@@ -235,7 +235,7 @@ class KVpopCache:
 
 
 def topk_cutoff(prio, n_sink: int, window: int, k: int, lengths=None, rank=None, tau=None,
-                stream=None):
+                order=None, stream=None):
     """Static ranks and running top-k cutoffs of each row of ``prio [n_rows][S]`` (fp32, CUDA)."""
     n_rows, S = prio.shape
     dev = prio.device
@@ -244,12 +244,12 @@ def topk_cutoff(prio, n_sink: int, window: int, k: int, lengths=None, rank=None,
     nb = int(kvpop_topk_workspace_bytes(n_rows, S))
     ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=dev)
     _ck(kvpop_topk_cutoff(_ptr(prio), _ptr(lengths), n_rows, S, n_sink, window, k, _ptr(rank),
-                          _ptr(tau), _ptr(ws), nb, _stream(stream)), "kvpop_topk_cutoff")
+                          _ptr(tau), _ptr(order), _ptr(ws), nb, _stream(stream)), "kvpop_topk_cutoff")
     return rank, tau
 
 
 def prompt_attention(Q, K, V, rank, tau, n_sink: int, window: int, k: int, lengths=None, Y=None,
-                     lse=None, want_lse: bool = True, stream=None):
+                     lse=None, want_lse: bool = True, order=None, stream=None):
     """Masked causal attention under the running top-k mask.  ``Q [n][H*G][S][d]``,
     ``K, V [n][H][S][d]``, ``rank, tau [n][H][S]``; returns (Y fp32, LSE fp32 or None)."""
     n_seq, H, S, d = K.shape
@@ -258,7 +258,8 @@ def prompt_attention(Q, K, V, rank, tau, n_sink: int, window: int, k: int, lengt
     Y = torch.empty((n_seq, H * G, S, d), dtype=torch.float32, device=dev) if Y is None else Y
     if lse is None and want_lse:
         lse = torch.empty((n_seq, H * G, S), dtype=torch.float32, device=dev)
-    _ck(kvpop_prompt_attention(_ptr(Q), _ptr(K), _ptr(V), _ptr(rank), _ptr(tau), _ptr(lengths), n_seq,
+    _ck(kvpop_prompt_attention(_ptr(Q), _ptr(K), _ptr(V), _ptr(rank), _ptr(tau), _ptr(order),
+                               _ptr(lengths), n_seq,
                                H, G, d, S, n_sink, window, k, dtype_code(K.dtype), _ptr(Y), _ptr(lse),
                                _stream(stream)), "kvpop_prompt_attention")
     return Y, lse

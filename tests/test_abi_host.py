@@ -93,17 +93,19 @@ def test_topk_and_prompt_attention_reject_bad_arguments(kv):
     assert kv.kvpop_topk_workspace_bytes(0, 100) == 0
     ok, bad, align = 0, 1, 2          # KVPOP_OK, KVPOP_ERR_INVALID_ARG, KVPOP_ERR_ALIGN
     cut = kv.kvpop_topk_cutoff
-    assert cut(P, None, 0, 100, 0, 4, 8, P, P, P, ws, None) == ok          # nothing to do
-    assert cut(P, None, 4, 100, 0, 0, 8, P, P, P, ws, None) == bad         # window 0
-    assert cut(P, None, 4, 100, 0, 4, 0, P, P, P, ws, None) == bad         # k 0
-    assert cut(P, None, 4, (1 << 18) + 1, 0, 4, 8, P, P, P, ws, None) == bad
-    assert cut(P, None, 4, 100, 0, 4, 8, P, P, P, ws - 1, None) == bad     # workspace too small
-    assert cut(None, None, 4, 100, 0, 4, 8, P, P, P, ws, None) == bad
-    assert cut(P + 2, None, 4, 100, 0, 4, 8, P, P, P, ws, None) == align
-    assert cut(P, None, 4, 100, 0, 4, 8, P, P, P + 16, ws, None) == align  # workspace 256-aligned
+    assert cut(P, None, 0, 100, 0, 4, 8, P, P, None, P, ws, None) == ok          # nothing to do
+    assert cut(P, None, 4, 100, 0, 0, 8, P, P, None, P, ws, None) == bad         # window 0
+    assert cut(P, None, 4, 100, 0, 4, 0, P, P, None, P, ws, None) == bad         # k 0
+    assert cut(P, None, 4, (1 << 18) + 1, 0, 4, 8, P, P, None, P, ws, None) == bad
+    assert cut(P, None, 4, 100, 0, 4, 8, P, P, None, P, ws - 1, None) == bad     # workspace too small
+    assert cut(None, None, 4, 100, 0, 4, 8, P, P, None, P, ws, None) == bad
+    assert cut(P + 2, None, 4, 100, 0, 4, 8, P, P, None, P, ws, None) == align
+    assert cut(P, None, 4, 100, 0, 4, 8, P, P, P + 2, P, ws, None) == align      # order 4-aligned
+    assert cut(P, None, 4, 100, 0, 4, 8, P, P, None, P + 16, ws, None) == align  # workspace 256-aligned
     att = kv.kvpop_prompt_attention
     args = lambda **o: [o.get(n, v) for n, v in (
-        ("Q", P), ("K", P), ("V", P), ("rank", P), ("tau", P), ("len", None), ("n", 2), ("H", 8),
+        ("Q", P), ("K", P), ("V", P), ("rank", P), ("tau", P), ("order", None), ("len", None),
+        ("n", 2), ("H", 8),
         ("G", 4), ("d", 128), ("S", 64), ("s", 0), ("w", 16), ("k", 64), ("dt", kv.KVPOP_BF16),
         ("Y", P), ("lse", P), ("st", None))]
     assert att(*args(n=0)) == ok
@@ -117,6 +119,7 @@ def test_topk_and_prompt_attention_reject_bad_arguments(kv):
     assert att(*args(Q=P + 8)) == align
     assert att(*args(Y=P + 4)) == align
     assert att(*args(lse=P + 2)) == align
+    assert att(*args(order=P + 2)) == align
 
 
 def test_causal_lse_and_future_target_reject_bad_arguments(kv):

@@ -55,14 +55,18 @@ def test_topk_cutoff_bitexact(cuda_device, s, w, k, levels):
     lengths = [3000, 2999, 1, 0, 1500, 2055]
     prio = plant_specials(gen.uniform_scores(7, STREAM_PRIO, (len(lengths), S), levels=levels))
     L = torch.tensor(lengths, dtype=torch.int32, device=cuda_device)
-    rank, tau = kv().topk_cutoff(prio.to(cuda_device), s, w, k, lengths=L)
-    rank, tau = rank.cpu().numpy(), tau.cpu().numpy()
+    order = torch.full((len(lengths), S), -7, dtype=torch.int32, device=cuda_device)
+    rank, tau = kv().topk_cutoff(prio.to(cuda_device), s, w, k, lengths=L, order=order)
+    rank, tau, order = rank.cpu().numpy(), tau.cpu().numpy(), order.cpu().numpy()
     for r, n in enumerate(lengths):
         want_rank = rt.static_ranks(prio[r, :n].numpy())
         want_tau = rt.fenwick_cutoffs(want_rank, s, w, k)
         assert np.array_equal(rank[r, :n], want_rank), f"row {r}: ranks differ"
         assert np.array_equal(tau[r, :n], want_tau), f"row {r}: cutoffs differ"
         assert np.all(rank[r, n:] == -1) and np.all(tau[r, n:] == -1)
+        # order is the inverse permutation of the ranks; entries past the length untouched
+        assert np.array_equal(order[r, want_rank], np.arange(n)), f"row {r}: order differs"
+        assert np.all(order[r, n:] == -7)
 
 
 def test_topk_cutoff_longest_rows(cuda_device):
@@ -95,17 +99,30 @@ def attention_case(cfg, lengths, s, w, k, seed_prio, device):
     return Q, K, V, ranks, taus
 
 
+def inverse_ranks(ranks, lengths):
+    """Positions by rank, built from the oracle's ranks (the order a rank walk reads)."""
+    order = np.full(ranks.shape, -1, dtype=np.int32)
+    for b, n in enumerate(lengths):
+        for h in range(ranks.shape[1]):
+            order[b, h, ranks[b, h, :n]] = np.arange(n, dtype=np.int32)
+    return order
+
+
 @pytest.mark.parametrize("dtype,d,G", [("f32", 64, 2), ("f32", 128, 4), ("bf16", 128, 4),
                                        ("bf16", 64, 2), ("bf16", 128, 1)])
-def test_prompt_attention_matches_oracle(cuda_device, dtype, d, G):
+@pytest.mark.parametrize("by_rank", [False, True])
+def test_prompt_attention_matches_oracle(cuda_device, dtype, d, G, by_rank):
+    """Masked attention against the oracle; with ``by_rank`` the key lists of the late
+    tiles are built by walking the ranks up to the tile's largest cutoff."""
     cfg = get_config("tiny").with_(kv_dtype=dtype, head_dim=d, q_per_kv=G, n_kv_heads=2, batch=2)
     lengths = [300, 237]
     s, w, k = 2, 5, 40
     Q, K, V, ranks, taus = attention_case(cfg, lengths, s, w, k, 3, cuda_device)
     dev = cuda_device
     L = torch.tensor(lengths, dtype=torch.int32, device=dev)
+    order = torch.from_numpy(inverse_ranks(ranks, lengths)).to(dev) if by_rank else None
     Y, lse = kv().prompt_attention(Q.to(dev), K.to(dev), V.to(dev), torch.from_numpy(ranks).to(dev),
-                                   torch.from_numpy(taus).to(dev), s, w, k, lengths=L)
+                                   torch.from_numpy(taus).to(dev), s, w, k, lengths=L, order=order)
     Y, lse = Y.cpu().numpy(), lse.cpu().numpy()
     ey = el = 0.0
     for b, n in enumerate(lengths):
@@ -114,7 +131,7 @@ def test_prompt_attention_matches_oracle(cuda_device, dtype, d, G):
                                        f64(V[b, h, :n]), ranks[b, h, :n], taus[b, h, :n], s, w)
             ey = max(ey, float(np.abs(Y[b, h * G:(h + 1) * G, :n] - y).max()))
             el = max(el, float(np.abs(lse[b, h * G:(h + 1) * G, :n] - l).max()))
-    print(f"prompt attention {dtype} d{d} G{G}: max-abs y {ey:.2e}, lse {el:.2e}")
+    print(f"prompt attention {dtype} d{d} G{G} by_rank={by_rank}: max-abs y {ey:.2e}, lse {el:.2e}")
     assert ey <= Y_TOL[dtype] and el <= LSE_TOL[dtype]
 
 
@@ -130,10 +147,17 @@ def run_prefill_attend(cache, cfg, lengths, device, override, b0=0, want=True):
     lse = torch.empty((n, HG, S), dtype=torch.float32, device=device)
     rank = torch.empty((n, H, S), dtype=torch.int32, device=device)
     tau = torch.empty((n, H, S), dtype=torch.int32, device=device)
+    order = torch.full((n, H, S), -7, dtype=torch.int32, device=device)
     ov = None if override is None else override[b0:b0 + n, :, :S].contiguous()
-    cache.prefill_attend(Q, K, V, lengths, Y, lse, first_seq=b0, override=ov, rank=rank, tau=tau)
+    cache.prefill_attend(Q, K, V, lengths, Y, lse, first_seq=b0, override=ov, rank=rank, tau=tau,
+                         order=order)
     torch.cuda.synchronize()
     cache.check()
+    rk, od = rank.cpu().numpy(), order.cpu().numpy()
+    for b, P in enumerate(lengths):
+        for h in range(H):
+            assert np.array_equal(od[b, h, rk[b, h, :P]], np.arange(P)), (b, h)
+            assert np.all(od[b, h, P:] == -7), (b, h)
     return Y, lse, rank, tau
 
 
