@@ -420,9 +420,20 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
       tmem_ld32(tS + b2 * T6_BN, *reinterpret_cast<float(*)[32]>(s));
       tmem_ld32(tS + b2 * T6_BN + 32, *reinterpret_cast<float(*)[32]>(s + 32));
       tmem_wait_ld();
+      // log2-unit logits less the queries' normalisers, two at a time (packed fp32 FMA);
       // the stage's query rows and LSE are no longer needed once read
+      {
+        const float4* l4 = reinterpret_cast<const float4*>(lseS + st * T6_BN);
 #pragma unroll
-      for (int i = 0; i < 64; ++i) s[i] = fmaf(s[i], c2, -lseS[st * T6_BN + i] * kLog2e);
+        for (int i4 = 0; i4 < 16; ++i4) {
+          const float4 v = l4[i4];
+          const uint64_t nl01 = f2_mul(f2_pack(v.x, v.y), f2_pack(-kLog2e, -kLog2e));
+          const uint64_t nl23 = f2_mul(f2_pack(v.z, v.w), f2_pack(-kLog2e, -kLog2e));
+          f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), f2_pack(c2, c2), nl01), s[4 * i4], s[4 * i4 + 1]);
+          f2_unpack(f2_fma(f2_pack(s[4 * i4 + 2], s[4 * i4 + 3]), f2_pack(c2, c2), nl23), s[4 * i4 + 2],
+                    s[4 * i4 + 3]);
+        }
+      }
       fence_before();
       mbar_arrive(bar(T6_EMPTY + st));
       mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
@@ -434,21 +445,33 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
           if (d < t + w || d > hi) s[i] = -INFINITY;
         }
       }
+      // row maximum: 8 chains of three-input maxima
       float pm[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) pm[k] = s[k];
 #pragma unroll
-      for (int i = 8; i < 64; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      for (int i = 8; i < 64; i += 16)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+      const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
       const float mn = fmaxf(m, mx);
       const float base = mn == -INFINITY ? 0.f : mn;
-      float ps[8];
+      // sum of 2^(x - base), differences and partial sums packed in pairs
+      const uint64_t nb = f2_pack(-base, -base);
+      uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+      for (int i = 0; i < 64; i += 8) {
 #pragma unroll
-      for (int i = 0; i < 64; ++i) ps[i & 7] += ex2(s[i] - base);
-      l = l * ex2(m - base) + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
+        for (int k = 0; k < 4; ++k) {
+          float x0, x1;
+          f2_unpack(f2_add(f2_pack(s[i + 2 * k], s[i + 2 * k + 1]), nb), x0, x1);
+          ps[k] = f2_add(ps[k], f2_pack(ex2(x0), ex2(x1)));
+        }
+      }
+      float q[8];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) f2_unpack(ps[k], q[2 * k], q[2 * k + 1]);
+      l = l * ex2(m - base) + (((q[0] + q[1]) + (q[2] + q[3])) + ((q[4] + q[5]) + (q[6] + q[7])));
       m = mn;
       if (b == nblk - 1) {                          // head g done: write and reset
         if (t <= t1) a.logm[(qrow0 + g) * S + t] = l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
