@@ -235,14 +235,15 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
             }
           }
         }
-        // 8 independent partial maxima (a 64-long chain would serialise on latency)
+        // 8 independent chains of three-input maxima (one 64-long chain would serialise)
         float pm[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) pm[k] = s[k];
 #pragma unroll
-        for (int i = 8; i < 64; ++i) pm[i & 7] = fmaxf(pm[i & 7], s[i]);
-        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+        for (int i = 8; i < 64; i += 16)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+        const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
         const float mxs = mx * c2;                  // row maximum, log2 units
         float alpha = 1.f, m_new = m;
         bool resc = false;
@@ -252,14 +253,23 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
           resc = m != -INFINITY;
         }
         const float base = m_new == -INFINITY ? 0.f : m_new;
+        // probabilities 2^(s c2 - base): scale-and-shift and the partial sums in packed pairs
+        const uint64_t cc = f2_pack(c2, c2), nb = f2_pack(-base, -base);
+        uint64_t ps2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+        for (int i = 0; i < 64; i += 8) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(s[i + 2 * k], s[i + 2 * k + 1]), cc, nb), x0, x1);
+            s[i + 2 * k] = ex2(x0);
+            s[i + 2 * k + 1] = ex2(x1);
+            ps2[k] = f2_add(ps2[k], f2_pack(s[i + 2 * k], s[i + 2 * k + 1]));
+          }
+        }
         float ps[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) ps[k] = 0.f;
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          s[i] = ex2(fmaf(s[i], c2, -base));
-          ps[i & 7] += s[i];
-        }
+        for (int k = 0; k < 4; ++k) f2_unpack(ps2[k], ps[2 * k], ps[2 * k + 1]);
         const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
         l = l * alpha + sum;
         m = m_new;
