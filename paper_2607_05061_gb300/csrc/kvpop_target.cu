@@ -284,8 +284,8 @@ __global__ void __launch_bounds__(TgP<HD>::THREADS, 1) target_tc_kernel(TargetAr
 // ---------------------------------------------------------------- tcgen05 kernel (d = 128)
 constexpr int T6_HALF = 128;
 constexpr int T6_ROWS = 2 * T6_HALF;            // keys per CTA
-constexpr int T6_BN = 64;                       // queries per block
-constexpr int T6_ST = 8;                        // query-block stages
+constexpr int T6_BN = 128;                      // queries per block (MMA N)
+constexpr int T6_ST = 4;                        // query-block stages
 constexpr int T6_MMA_WARP = 8;                  // warps 0-7 softmax, 8 MMA, 9-11 producers
 constexpr int T6_PT = 96;
 constexpr int T6_THREADS = 32 * 12;
@@ -336,7 +336,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
     mbar_init(bar(T6_KFULL), T6_PT);
     mbar_fence_init();
   }
-  if (warp == T6_MMA_WARP) tmem_alloc(sb + T6_OFF_TMEM, 256);
+  if (warp == T6_MMA_WARP) tmem_alloc(sb + T6_OFF_TMEM, 512);
   fence_before();
   __syncthreads();
   fence_after();
@@ -364,9 +364,9 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         const bool ok = d0 + r <= d_hi;
         cp_async16(qd + tile_off(r, c, T6_BN), Qg + (size_t)(ok ? d0 + r : d0) * 128 + c * 8, ok ? 16 : 0);
       }
-      if (pt < T6_BN) {
+      for (int i = pt; i < T6_BN; i += T6_PT) {
         const float* lse = a.lse + (qrow0 + g) * S;
-        cp_async4(sb + T6_OFF_LSE + (st * T6_BN + pt) * 4, lse + min(d0 + pt, d_hi));
+        cp_async4(sb + T6_OFF_LSE + (st * T6_BN + i) * 4, lse + min(d0 + i, d_hi));
       }
       cp_async_arrive_noinc(bar(T6_FULL + st));
     }
@@ -388,7 +388,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
           if (j >= 2 && !(ok = mbar_wait(bar(T6_PFULL + 2 * hh + b2), ((j - 2) >> 1) & 1, a.err, T6ERR_WAIT)))
             break;
           fence_after();
-          const uint32_t dS = tmem + hh * 128 + (uint32_t)b2 * T6_BN;
+          const uint32_t dS = tmem + hh * 256 + (uint32_t)b2 * T6_BN;
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks)
             mma_bf16(dS, kmajor_desc(sb + hh * T6_KB, T6_HALF, ks), kmajor_desc(qb, T6_BN, ks), idS, ks > 0);
@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
     const int r = (warp & 3) * 32 + lane;
     const int t = t0 + hh * T6_HALF + r;
     const int hi = t <= t1 ? future_hi(t, L, w, la) : -1;
-    const uint32_t tS = tmem + ((uint32_t)((warp & 3) * 32) << 16) + hh * 128;
+    const uint32_t tS = tmem + ((uint32_t)((warp & 3) * 32) << 16) + hh * 256;
     const float* lseS = reinterpret_cast<const float*>(sm6 + T6_OFF_LSE);
     const float c2 = a.kscale;
     float m = -INFINITY, l = 0.f;
@@ -416,63 +416,71 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
       const int d0 = d_lo + b * T6_BN;
       if (!uniform(mbar_wait(bar(T6_SFULL + 2 * hh + b2), (j >> 1) & 1, a.err, T6ERR_WAIT))) break;
       fence_after();
-      float s[64];
-      tmem_ld32(tS + b2 * T6_BN, *reinterpret_cast<float(*)[32]>(s));
-      tmem_ld32(tS + b2 * T6_BN + 32, *reinterpret_cast<float(*)[32]>(s + 32));
-      tmem_wait_ld();
-      // log2-unit logits less the queries' normalisers, two at a time (packed fp32 FMA);
-      // the stage's query rows and LSE are no longer needed once read
-      {
-        const float4* l4 = reinterpret_cast<const float4*>(lseS + st * T6_BN);
+      // the block's 128 columns as two 64-column halves, each folded into the running sum
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        const int e0 = d0 + 64 * c;
+        float s[64];
+        tmem_ld32(tS + b2 * T6_BN + 64 * c, *reinterpret_cast<float(*)[32]>(s));
+        tmem_ld32(tS + b2 * T6_BN + 64 * c + 32, *reinterpret_cast<float(*)[32]>(s + 32));
+        tmem_wait_ld();
+        // log2-unit logits less the queries' normalisers, two at a time (packed fp32 FMA)
+        {
+          const float4* l4 = reinterpret_cast<const float4*>(lseS + st * T6_BN + 64 * c);
 #pragma unroll
-        for (int i4 = 0; i4 < 16; ++i4) {
-          const float4 v = l4[i4];
-          const uint64_t nl01 = f2_mul(f2_pack(v.x, v.y), f2_pack(-kLog2e, -kLog2e));
-          const uint64_t nl23 = f2_mul(f2_pack(v.z, v.w), f2_pack(-kLog2e, -kLog2e));
-          f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), f2_pack(c2, c2), nl01), s[4 * i4], s[4 * i4 + 1]);
-          f2_unpack(f2_fma(f2_pack(s[4 * i4 + 2], s[4 * i4 + 3]), f2_pack(c2, c2), nl23), s[4 * i4 + 2],
-                    s[4 * i4 + 3]);
+          for (int i4 = 0; i4 < 16; ++i4) {
+            const float4 v = l4[i4];
+            const uint64_t nl01 = f2_mul(f2_pack(v.x, v.y), f2_pack(-kLog2e, -kLog2e));
+            const uint64_t nl23 = f2_mul(f2_pack(v.z, v.w), f2_pack(-kLog2e, -kLog2e));
+            f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), f2_pack(c2, c2), nl01), s[4 * i4],
+                      s[4 * i4 + 1]);
+            f2_unpack(f2_fma(f2_pack(s[4 * i4 + 2], s[4 * i4 + 3]), f2_pack(c2, c2), nl23), s[4 * i4 + 2],
+                      s[4 * i4 + 3]);
+          }
         }
-      }
-      fence_before();
-      mbar_arrive(bar(T6_EMPTY + st));
-      mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
-      const bool masked = d0 < t1 + w || d0 + T6_BN - 1 > d_hi || (la > 0 && d0 + T6_BN - 1 > t0 + w + la);
-      if (masked) {
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          const int d = d0 + i;
-          if (d < t + w || d > hi) s[i] = -INFINITY;
+        if (c == 1) {
+          // the stage's query rows and LSE, and the S buffer, are no longer needed
+          fence_before();
+          mbar_arrive(bar(T6_EMPTY + st));
+          mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
         }
-      }
-      // row maximum: 8 chains of three-input maxima
-      float pm[8];
+        const bool masked = e0 < t1 + w || e0 + 63 > d_hi || (la > 0 && e0 + 63 > t0 + w + la);
+        if (masked) {
 #pragma unroll
-      for (int k = 0; k < 8; ++k) pm[k] = s[k];
-#pragma unroll
-      for (int i = 8; i < 64; i += 16)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
-      const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
-      const float mn = fmaxf(m, mx);
-      const float base = mn == -INFINITY ? 0.f : mn;
-      // sum of 2^(x - base), differences and partial sums packed in pairs
-      const uint64_t nb = f2_pack(-base, -base);
-      uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-      for (int i = 0; i < 64; i += 8) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          float x0, x1;
-          f2_unpack(f2_add(f2_pack(s[i + 2 * k], s[i + 2 * k + 1]), nb), x0, x1);
-          ps[k] = f2_add(ps[k], f2_pack(ex2(x0), ex2(x1)));
+          for (int i = 0; i < 64; ++i) {
+            const int d = e0 + i;
+            if (d < t + w || d > hi) s[i] = -INFINITY;
+          }
         }
-      }
-      float q[8];
+        // row maximum: 8 chains of three-input maxima
+        float pm[8];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) f2_unpack(ps[k], q[2 * k], q[2 * k + 1]);
-      l = l * ex2(m - base) + (((q[0] + q[1]) + (q[2] + q[3])) + ((q[4] + q[5]) + (q[6] + q[7])));
-      m = mn;
+        for (int k = 0; k < 8; ++k) pm[k] = s[k];
+#pragma unroll
+        for (int i = 8; i < 64; i += 16)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+        const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
+        const float mn = fmaxf(m, mx);
+        const float base = mn == -INFINITY ? 0.f : mn;
+        // sum of 2^(x - base), differences and partial sums packed in pairs
+        const uint64_t nb = f2_pack(-base, -base);
+        uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+        for (int i = 0; i < 64; i += 8) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            float x0, x1;
+            f2_unpack(f2_add(f2_pack(s[i + 2 * k], s[i + 2 * k + 1]), nb), x0, x1);
+            ps[k] = f2_add(ps[k], f2_pack(ex2(x0), ex2(x1)));
+          }
+        }
+        float q[8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) f2_unpack(ps[k], q[2 * k], q[2 * k + 1]);
+        l = l * ex2(m - base) + (((q[0] + q[1]) + (q[2] + q[3])) + ((q[4] + q[5]) + (q[6] + q[7])));
+        m = mn;
+      }
       if (b == nblk - 1) {                          // head g done: write and reset
         if (t <= t1) a.logm[(qrow0 + g) * S + t] = l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
         m = -INFINITY;
@@ -482,7 +490,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
   }
   fence_before();
   __syncthreads();
-  if (warp == T6_MMA_WARP) tmem_dealloc(tmem, 256);
+  if (warp == T6_MMA_WARP) tmem_dealloc(tmem, 512);
 }
 
 // ---------------------------------------------------------------- aggregation
