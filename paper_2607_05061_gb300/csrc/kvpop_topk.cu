@@ -233,9 +233,11 @@ __global__ void cutoff_kernel(CutArgs a, int chunk) {
   const int L = row_length(a.len, a.rows_per_len, row, S);
   const int32_t* rank = a.rank + (size_t)row * S;
   int32_t* tau_out = a.tau + (size_t)row * S;
-  if (warp == 0)
+  if (warp == 0 && blockIdx.y == 0)
     for (int i = L + lane; i < S; i += 32) tau_out[i] = -1;
-  const int qa = warp * chunk;
+  // chunk blockIdx.y * warps + warp of the row: the row's chunks are spread over
+  // gridDim.y CTAs so that short batches still fill the GPU
+  const int qa = (blockIdx.y * (blockDim.x >> 5) + warp) * chunk;
   if (qa >= L) return;
   const int qb = min(qa + chunk, L);
   uint32_t* bits = bitsets + (size_t)warp * words;
@@ -310,12 +312,17 @@ cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len,
   // chunks per row: up to 16 warps, each with its own bitset of S bits in shared memory
   const size_t words_bytes = (size_t)((S + 31) / 32) * 4;
   const int nch = (int)std::max<size_t>(1, std::min<size_t>(CUT_MAX_WARPS, (200 * 1024) / words_bytes));
-  const int chunk = (S + nch - 1) / nch;
+  // CTAs per row: enough for about two per SM, while every chunk keeps >= 512 queries
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int want = std::max(1, (2 * sms + n_rows - 1) / n_rows);
+  const int split = std::max(1, std::min(want, S / (nch * 512)));
+  const int chunk = (S + nch * split - 1) / (nch * split);
   const size_t smem = (size_t)nch * words_bytes;
   e = cudaFuncSetAttribute(cutoff_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   CutArgs ca{rank, len, rows_per_len, n_rows, S, s, w, k, tau};
-  cutoff_kernel<<<n_rows, nch * 32, smem, stream>>>(ca, chunk);
+  cutoff_kernel<<<dim3(n_rows, split), nch * 32, smem, stream>>>(ca, chunk);
   return cudaGetLastError();
 }
 
