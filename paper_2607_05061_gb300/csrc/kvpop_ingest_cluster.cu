@@ -68,6 +68,16 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
                : "memory");
 }
 
+// D (16x8, fp32) += A (16x8, tf32, row) B (8x8, tf32, col), legacy tensor-core MMA
+__device__ __forceinline__ void mma_tf32_16x8x8(float (&c)[4], const uint32_t (&a)[4],
+                                                const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7},"
+      " {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
 struct ClLayout {              // byte offsets into dynamic shared memory
   int ws, x, qm, qrow, ring, newkv, part, total;
 };
@@ -77,7 +87,7 @@ __host__ __device__ inline ClLayout cl_layout(int d, int D, int G, int FS, int e
   int o = 0;
   L.ws = o;    o += 3 * d * FS * 4;                 // W1 slice, then b1, w2 slices
   o += 2 * FS * 4;
-  L.x = o;     o += SBC * 3 * d * 4;                // scorer inputs of the 16 sequences
+  L.x = o;     o += SBC * (3 * d + 4) * 4;          // scorer inputs of the 16 sequences (row stride 3d + 4)
   L.qm = o;    o += OWN * D * d * 4;                // window query means of the owned sequences
   L.qrow = o;  o += OWN * G * R;                    // new queries
   L.ring = o;  o += OWN * 2 * R;                    // K, V row of the leaving token
@@ -103,7 +113,8 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
   float* Ws = reinterpret_cast<float*>(smem + L.ws);
   const float* b1s = Ws + in_dim * FS;
   const float* w2s = b1s + FS;
-  float* X = reinterpret_cast<float*>(smem + L.x);           // [SBC][3d]
+  float* X = reinterpret_cast<float*>(smem + L.x);           // [SBC][3d + 4]
+  const int XS = in_dim + 4;
   float* rqm = reinterpret_cast<float*>(smem + L.qm);        // [OWN][D][d]
   T* qrow = reinterpret_cast<T*>(smem + L.qrow);             // [OWN][G][d]
   T* ring = reinterpret_cast<T*>(smem + L.ring);             // [OWN][2][d]
@@ -215,7 +226,7 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
     const int ri = p >= 0 ? p % D : 0;
     const T* ku = ring + (size_t)(2 * o) * d;                 // the leaving token u = p - D
     const T* vu = ring + (size_t)(2 * o + 1) * d;
-    const uint32_t xrow = smem_u32(X + (size_t)j * in_dim);
+    const uint32_t xrow = smem_u32(X + (size_t)j * XS);
     const int nq4 = in_dim / 16;             // float4s per quarter
     if (lane < nq4) {
       const int i4 = qq * nq4 + lane;
@@ -268,35 +279,86 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
   cluster_sync();   // every X row is in every CTA
 
   // ---- this CTA's hidden slice for all 16 sequences --------------------------------------
-  // Thread (f, ks) accumulates hidden unit f over input slice ks for every sequence: per
-  // 4 inputs, 4 weights and 16 broadcast input vectors feed 64 FMAs.  The slices' partial
-  // sums meet in shared memory (over the input rows, no longer needed), then warp w adds
-  // b1, applies the activation and contracts with w2 for sequences 2w, 2w+1.
+  // H[16 sequences][FS] = X W, fp32-accurate.  With FS a multiple of 8 it runs on the tensor
+  // pipe: m16n8k8 tf32 MMAs, each operand split into a tf32 head and its residual and
+  // X W = X_hi W_hi + X_hi W_lo + X_lo W_hi (the dropped X_lo W_lo is below fp32 rounding);
+  // warp w takes k-steps [w K8 / 8, (w + 1) K8 / 8) of the 3d inputs.  Otherwise thread
+  // (f, ks) accumulates unit f over input slice ks for every sequence.  Either way the
+  // partial sums meet in shared memory (over the input rows, no longer needed), then warp w
+  // adds b1, applies the activation and contracts with w2 for sequences 2w, 2w+1.
   {
-    // input slices (FS <= 64); NKS * FS <= 3d keeps the partial sums inside the input rows
-    const int NKS = min(NT / FS, in_dim / FS);
-    const int SL = ((in_dim + NKS - 1) / NKS + 3) & ~3;   // inputs per slice, multiple of 4
-    const int f = tid % FS, ks = tid / FS;
-    float acc[SBC];
+    // (the 8 warp partials of [16][FS] must fit in the input rows: 8 FS <= 3d + 4)
+    const bool tc = (FS % 8) == 0 && (in_dim % 64) == 0 && 8 * FS <= XS && FS <= 64;
+    int NKS;                                          // partial sums per (sequence, unit)
+    float* red = X;                                   // [NKS][SBC][FS]
+    if (tc) {
+      NKS = NT / 32;
+      const int g = lane >> 2, tig = lane & 3;
+      const int k8 = in_dim / 8, kper = k8 / NKS, kb = warp * kper;
+      float acc[8][4];                                // up to FS = 64: 8 n-tiles
 #pragma unroll
-    for (int j = 0; j < SBC; ++j) acc[j] = 0.f;
-    if (ks < NKS) {
-      const int i_end = min(in_dim, (ks + 1) * SL);
-      for (int i = ks * SL; i < i_end; i += 4) {
-        const float w0 = Ws[(i + 0) * FS + f], w1 = Ws[(i + 1) * FS + f];
-        const float w2 = Ws[(i + 2) * FS + f], w3 = Ws[(i + 3) * FS + f];
+      for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
-        for (int j = 0; j < SBC; ++j) {
-          const float4 u = *reinterpret_cast<const float4*>(X + (size_t)j * in_dim + i);
-          acc[j] = fmaf(u.x, w0, fmaf(u.y, w1, fmaf(u.z, w2, fmaf(u.w, w3, acc[j]))));
+        for (int e = 0; e < 4; ++e) acc[nt][e] = 0.f;
+      auto split = [](float x, uint32_t& hi, uint32_t& lo) {
+        asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+        lo = __float_as_uint(x - __uint_as_float(hi));
+      };
+      for (int kk = 0; kk < kper; ++kk) {
+        const int k0 = (kb + kk) * 8;
+        uint32_t ah[4], al[4];
+        split(X[(size_t)g * XS + k0 + tig], ah[0], al[0]);
+        split(X[(size_t)(g + 8) * XS + k0 + tig], ah[1], al[1]);
+        split(X[(size_t)g * XS + k0 + tig + 4], ah[2], al[2]);
+        split(X[(size_t)(g + 8) * XS + k0 + tig + 4], ah[3], al[3]);
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+          if (nt * 8 >= FS) break;
+          uint32_t bh[2], bl[2];
+          split(Ws[(size_t)(k0 + tig) * FS + nt * 8 + g], bh[0], bl[0]);
+          split(Ws[(size_t)(k0 + tig + 4) * FS + nt * 8 + g], bh[1], bl[1]);
+          mma_tf32_16x8x8(acc[nt], ah, bh);
+          mma_tf32_16x8x8(acc[nt], ah, bl);
+          mma_tf32_16x8x8(acc[nt], al, bh);
         }
       }
-    }
-    __syncthreads();                                  // every thread is done with X
-    float* red = X;                                   // [NKS][SBC][FS] partial sums
-    if (ks < NKS) {
+      __syncthreads();                                // every warp is done with X
 #pragma unroll
-      for (int j = 0; j < SBC; ++j) red[((size_t)ks * SBC + j) * FS + f] = acc[j];
+      for (int nt = 0; nt < 8; ++nt) {
+        if (nt * 8 >= FS) break;
+        const int col = nt * 8 + 2 * tig;
+        float* r0 = red + ((size_t)warp * SBC + g) * FS + col;
+        float* r8 = red + ((size_t)warp * SBC + g + 8) * FS + col;
+        r0[0] = acc[nt][0];
+        r0[1] = acc[nt][1];
+        r8[0] = acc[nt][2];
+        r8[1] = acc[nt][3];
+      }
+    } else {
+      // NKS * FS <= 3d keeps the partial sums inside the input rows
+      NKS = min(NT / FS, in_dim / FS);
+      const int SL = ((in_dim + NKS - 1) / NKS + 3) & ~3;   // inputs per slice, multiple of 4
+      const int f = tid % FS, ks = tid / FS;
+      float acc[SBC];
+#pragma unroll
+      for (int j = 0; j < SBC; ++j) acc[j] = 0.f;
+      if (ks < NKS) {
+        const int i_end = min(in_dim, (ks + 1) * SL);
+        for (int i = ks * SL; i < i_end; i += 4) {
+          const float w0 = Ws[(i + 0) * FS + f], w1 = Ws[(i + 1) * FS + f];
+          const float w2 = Ws[(i + 2) * FS + f], w3 = Ws[(i + 3) * FS + f];
+#pragma unroll
+          for (int j = 0; j < SBC; ++j) {
+            const float4 u = *reinterpret_cast<const float4*>(X + (size_t)j * XS + i);
+            acc[j] = fmaf(u.x, w0, fmaf(u.y, w1, fmaf(u.z, w2, fmaf(u.w, w3, acc[j]))));
+          }
+        }
+      }
+      __syncthreads();                                // every thread is done with X
+      if (ks < NKS) {
+#pragma unroll
+        for (int j = 0; j < SBC; ++j) red[((size_t)ks * SBC + j) * FS + f] = acc[j];
+      }
     }
     __syncthreads();
     float c0 = 0.f, c1 = 0.f;
