@@ -288,8 +288,11 @@ kvpop_status kvpop_decode_step(kvpop_cache* cache, const void* q_dev, const void
                                float* score_out_dev, cudaStream_t stream);
 
 /* kvpop_decode_step on host buffers (pinned memory recommended): copies q/k/v
- * into library-owned device staging, runs the step and copies out back, all
- * on `stream` (the caller synchronises before reading out_host). */
+ * into library-owned device staging (one copy when k_host and v_host follow q_host
+ * directly in one buffer), runs the step and returns out, all on `stream` (the
+ * caller synchronises before reading out_host).  When out_host is pinned memory the
+ * device can address, the attention writes it directly; otherwise it is copied
+ * back from device staging. */
 kvpop_status kvpop_decode_step_host(kvpop_cache* cache, const void* q_host, const void* k_host,
                                     const void* v_host, float* out_host, cudaStream_t stream);
 

@@ -275,9 +275,13 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
   }
   ALLOC(part, float*, (size_t)2 * c->attend_grid * (dm.G * d + 2 * dm.G) * 4)
 #undef ALLOC
-  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * c->esz); c->stage_q = p; }
-  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_k = p; }
-  if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * d * c->esz); c->stage_v = p; }
+  // q | k | v staging in one block, so that adjacent host buffers take a single copy
+  if (s == KVPOP_OK) {
+    s = dev_alloc(c, &p, pairs * (dm.G + 2) * d * c->esz);
+    c->stage_q = p;
+    c->stage_k = static_cast<char*>(p) + pairs * dm.G * d * c->esz;
+    c->stage_v = static_cast<char*>(c->stage_k) + pairs * d * c->esz;
+  }
   if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * 4); c->stage_out = (float*)p; }
   if (s == KVPOP_OK && c->use_tc) {
     c->tc_maps.assign(tc_maps_size() + 64, 0);
@@ -680,13 +684,32 @@ kvpop_status kvpop_decode_step_host(kvpop_cache* c, const void* q, const void* k
   if (s != KVPOP_OK) return s;
   if (!q || !k || !v || !out) return KVPOP_ERR_INVALID_ARG;
   const size_t pairs = c->dm.pairs, d = c->dm.d, G = c->dm.G;
-  cudaError_t e = NOTE(cudaMemcpyAsync(c->stage_q, q, pairs * G * d * c->esz, cudaMemcpyHostToDevice, stream));
-  if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_k, k, pairs * d * c->esz, cudaMemcpyHostToDevice, stream));
-  if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_v, v, pairs * d * c->esz, cudaMemcpyHostToDevice, stream));
+  const size_t qb = pairs * G * d * c->esz, kb = pairs * d * c->esz;
+  const char* qc = static_cast<const char*>(q);
+  cudaError_t e = cudaErrorInvalidValue;
+  // adjacent buffers take one copy; adjacent addresses from different host allocations
+  // are refused by the runtime before anything is queued, and then take three
+  if (static_cast<const char*>(k) == qc + qb && static_cast<const char*>(v) == qc + qb + kb) {
+    e = cudaMemcpyAsync(c->stage_q, q, qb + 2 * kb, cudaMemcpyHostToDevice, stream);
+    if (e == cudaErrorInvalidValue) cudaGetLastError();
+  }
+  if (e == cudaErrorInvalidValue) {
+    e = NOTE(cudaMemcpyAsync(c->stage_q, q, qb, cudaMemcpyHostToDevice, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_k, k, kb, cudaMemcpyHostToDevice, stream));
+    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_v, v, kb, cudaMemcpyHostToDevice, stream));
+  }
   if (e != cudaSuccess) return poison_on(c, e);
-  s = kvpop_decode_step(c, c->stage_q, c->stage_k, c->stage_v, c->stage_out, nullptr, nullptr,
-                        nullptr, stream);
-  if (s != KVPOP_OK) return s;
+  // pinned host memory the device can address (NVLink-C2C / PCIe mapping) takes the
+  // attention output directly; anything else goes through the device staging buffer
+  cudaPointerAttributes pa{};
+  float* direct = nullptr;
+  if (cudaPointerGetAttributes(&pa, out) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+      pa.devicePointer != nullptr && aligned16(pa.devicePointer))
+    direct = static_cast<float*>(pa.devicePointer);
+  cudaGetLastError();   // a pointer the runtime does not know is not an error here
+  s = kvpop_decode_step(c, c->stage_q, c->stage_k, c->stage_v, direct ? direct : c->stage_out,
+                        nullptr, nullptr, nullptr, stream);
+  if (s != KVPOP_OK || direct) return s;
   e = NOTE(cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream));
   return poison_on(c, e);
 }
