@@ -15,11 +15,13 @@
 //
 // bf16 with d = 128 runs on the 5th-generation tensor cores (target_t5_kernel):
 // a CTA holds 256 keys as two 128-row A tiles in shared memory; producer warps
-// stream each head's query rows in blocks of 64 (with their LSE_d) through an
-// 8-stage cp.async ring; one thread issues S = K Q^T per half into a
-// tensor-memory double buffer; one softmax thread per (key, half) reads its row
-// with 32x32b loads and keeps the running max and sum.  The query rows are
-// contiguous, so the ring can run deep; the pass has no value half.
+// stream each head's query rows in blocks of 128 through a 4-stage cp.async ring
+// and store the block's -log2(e) LSE_d beside them; one thread issues S = K Q^T
+// per half into a tensor-memory double buffer; one softmax thread per (key,
+// half) reads its row with 32x32b loads.  s c - log2(e) LSE_d is the query's
+// log2 attention probability of the key, so the row's 2^x are summed with base 0
+// and a running maximum is taken only for a 64-column half whose sum leaves
+// [2^-60, 2^60].  The query rows are contiguous; the pass has no value half.
 //
 // Kernel 2 aggregates per KV head (Eq. 2, App. F.1-F.2):
 //   r_t = log(eps + Agg_g mbar_t^(g) / N_t),  N_t = max(1, S - (t + w)),
@@ -326,7 +328,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
   auto bar = [&](int i) { return sb + T6_OFF_BAR + 8u * (uint32_t)i; };
   if (tid == 0) {
     for (int i = 0; i < T6_ST; ++i) {
-      mbar_init(bar(T6_FULL + i), T6_PT);
+      mbar_init(bar(T6_FULL + i), 2 * T6_PT);            // cp.async arrivals + plain stores
       mbar_init(bar(T6_EMPTY + i), 1 + 2 * T6_HALF);   // MMA commit + every softmax thread (LSE)
     }
     for (int i = 0; i < 4; ++i) {
@@ -364,11 +366,12 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         const bool ok = d0 + r <= d_hi;
         cp_async16(qd + tile_off(r, c, T6_BN), Qg + (size_t)(ok ? d0 + r : d0) * 128 + c * 8, ok ? 16 : 0);
       }
-      for (int i = pt; i < T6_BN; i += T6_PT) {
-        const float* lse = a.lse + (qrow0 + g) * S;
-        cp_async4(sb + T6_OFF_LSE + (st * T6_BN + i) * 4, lse + min(d0 + i, d_hi));
-      }
+      // the block's queries' normalisers, stored once as -log2(e) LSE_d
+      float* nls = reinterpret_cast<float*>(sm6 + T6_OFF_LSE) + st * T6_BN;
+      const float* lse = a.lse + (qrow0 + g) * S;
+      for (int i = pt; i < T6_BN; i += T6_PT) nls[i] = -kLog2e * __ldg(lse + min(d0 + i, d_hi));
       cp_async_arrive_noinc(bar(T6_FULL + st));
+      mbar_arrive(bar(T6_FULL + st));
     }
     cp_wait<0>();
   } else if (warp == T6_MMA_WARP) {
@@ -397,6 +400,9 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         if (!ok) break;
         commit(bar(T6_EMPTY + st));
       }
+      // the last stage's release (the commit and the softmax) has landed before the CTA ends
+      if (ok && total > 0)
+        mbar_wait(bar(T6_EMPTY + (total - 1) % T6_ST), ((total - 1) / T6_ST) & 1, a.err, T6ERR_WAIT);
     }
     __syncwarp();
   } else {
@@ -406,7 +412,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
     const int t = t0 + hh * T6_HALF + r;
     const int hi = t <= t1 ? future_hi(t, L, w, la) : -1;
     const uint32_t tS = tmem + ((uint32_t)((warp & 3) * 32) << 16) + hh * 256;
-    const float* lseS = reinterpret_cast<const float*>(sm6 + T6_OFF_LSE);
+    const float* nlS = reinterpret_cast<const float*>(sm6 + T6_OFF_LSE);   // -log2(e) LSE_d per stage
     const float c2 = a.kscale;
     float m = -INFINITY, l = 0.f;
     auto uniform = [](bool x) { return __all_sync(0xffffffffu, x); };
@@ -415,6 +421,8 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
       const int g = j / nblk, b = j - g * nblk;
       const int d0 = d_lo + b * T6_BN;
       if (!uniform(mbar_wait(bar(T6_SFULL + 2 * hh + b2), (j >> 1) & 1, a.err, T6ERR_WAIT))) break;
+      // the stage's normalisers (complete long before S; the wait orders their reads)
+      if (!uniform(mbar_wait(bar(T6_FULL + st), (j / T6_ST) & 1, a.err, T6ERR_WAIT))) break;
       fence_after();
       // the block's 128 columns as two 64-column halves, each folded into the running sum
 #pragma unroll 1
@@ -424,32 +432,54 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         tmem_ld32(tS + b2 * T6_BN + 64 * c, *reinterpret_cast<float(*)[32]>(s));
         tmem_ld32(tS + b2 * T6_BN + 64 * c + 32, *reinterpret_cast<float(*)[32]>(s + 32));
         tmem_wait_ld();
-        // log2-unit logits less the queries' normalisers, two at a time (packed fp32 FMA)
-        {
-          const float4* l4 = reinterpret_cast<const float4*>(lseS + st * T6_BN + 64 * c);
-#pragma unroll
-          for (int i4 = 0; i4 < 16; ++i4) {
-            const float4 v = l4[i4];
-            const uint64_t nl01 = f2_mul(f2_pack(v.x, v.y), f2_pack(-kLog2e, -kLog2e));
-            const uint64_t nl23 = f2_mul(f2_pack(v.z, v.w), f2_pack(-kLog2e, -kLog2e));
-            f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), f2_pack(c2, c2), nl01), s[4 * i4],
-                      s[4 * i4 + 1]);
-            f2_unpack(f2_fma(f2_pack(s[4 * i4 + 2], s[4 * i4 + 3]), f2_pack(c2, c2), nl23), s[4 * i4 + 2],
-                      s[4 * i4 + 3]);
-          }
-        }
         if (c == 1) {
-          // the stage's query rows and LSE, and the S buffer, are no longer needed
+          // the S buffer is in registers: the MMA may overwrite it
           fence_before();
-          mbar_arrive(bar(T6_EMPTY + st));
           mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
         }
         const bool masked = e0 < t1 + w || e0 + 63 > d_hi || (la > 0 && e0 + 63 > t0 + w + la);
-        if (masked) {
+        if (masked) {                               // on the raw logits: -inf c2 + n = -inf
 #pragma unroll
           for (int i = 0; i < 64; ++i) {
             const int d = e0 + i;
             if (d < t + w || d > hi) s[i] = -INFINITY;
+          }
+        }
+        // x = s c2 - log2(e) LSE_d is the query's log2 attention probability of the key, so
+        // 2^x needs no running maximum unless the key lies outside the query's kept set
+        // with a much larger logit: sum with base 0, and take the maximum only when the
+        // half's sum leaves [2^-60, 2^60] (overflow, NaN, or every term tiny or masked).
+        // One loop forms x (packed FMA, kept in s for that case) and feeds the exponentials,
+        // so the FMA work issues under the MUFU's.
+        {
+          const float4* l4 = reinterpret_cast<const float4*>(nlS + st * T6_BN + 64 * c);
+          const uint64_t cc = f2_pack(c2, c2);
+          uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+          for (int i4 = 0; i4 < 16; ++i4) {
+            const float4 v = l4[i4];
+            f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), cc, f2_pack(v.x, v.y)), s[4 * i4],
+                      s[4 * i4 + 1]);
+            f2_unpack(f2_fma(f2_pack(s[4 * i4 + 2], s[4 * i4 + 3]), cc, f2_pack(v.z, v.w)), s[4 * i4 + 2],
+                      s[4 * i4 + 3]);
+            const int k = (2 * i4) & 3;
+            ps[k] = f2_add(ps[k], f2_pack(ex2(s[4 * i4]), ex2(s[4 * i4 + 1])));
+            ps[k + 1] = f2_add(ps[k + 1], f2_pack(ex2(s[4 * i4 + 2]), ex2(s[4 * i4 + 3])));
+          }
+          // the stage's query rows and normalisers are no longer needed
+          if (c == 1) mbar_arrive(bar(T6_EMPTY + st));
+          float q[8];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) f2_unpack(ps[k], q[2 * k], q[2 * k + 1]);
+          const float sum = ((q[0] + q[1]) + (q[2] + q[3])) + ((q[4] + q[5]) + (q[6] + q[7]));
+          if (sum >= 0x1p-60f && sum <= 0x1p60f) {
+            if (m <= 0.f) {                         // new base 0
+              l = (m == 0.f ? l : l * ex2(m)) + sum;
+              m = 0.f;
+            } else {
+              l = fmaf(sum, ex2(-m), l);
+            }
+            continue;
           }
         }
         // row maximum: 8 chains of three-input maxima
