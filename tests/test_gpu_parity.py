@@ -142,9 +142,10 @@ def test_planted_ties_bitexact(cuda_device):
     ("q4b", 256, [(0, 0), (3, 5), (7, 7)]),
     ("cr8x", 48, [(0, 0), (63, 7)]),
     ("ragged", 24, None),
+    ("q8b_stack", 24, [(0, 0), (31, 7)]),    # one layer of the 8B stack: b32, P=32768, B=8192
 ])
 def test_full_size_sampled(cuda_device, name, steps, sample):
-    cfg = get_config(name)
+    cfg = get_config(name, n_layers=1)
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
     if sample is None:   # shortest and longest sequence, and one below the budget
