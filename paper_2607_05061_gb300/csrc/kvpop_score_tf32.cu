@@ -16,7 +16,9 @@
 //    means (mean over the G heads) of the positions u0+1 .. u0+126+D and then
 //    average D of them per token, in the same order as the other kernels;
 //  * one thread loads the matching W1^T chunk (hi and lo, F rows x 32) by TMA
-//    and issues the 3 x 4 MMAs (M = 128, N = F, K = 8 each) per chunk;
+//    and issues the 3 x 4 MMAs (M = 128, N = F, K = 8 each) per chunk -- 2 x 4 for
+//    the k and v chunks of bf16 inputs, which are exact in tf32 (their lo is 0 and
+//    is not stored);
 //  * the builders finish: each thread reads half of its token's F pre-activations
 //    from tensor memory, adds b1, applies the activation, dots with w2, and one
 //    of the two halves writes the token's static priority.
@@ -176,9 +178,11 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
         fence_async_smem();
         fence_after();
         const uint32_t xb = sb + 2 * b * SC_XB, wb = sb + off.w + 2 * b * WB;
-        // products hi*hi, hi*lo, lo*hi
+        // products hi*hi, hi*lo, lo*hi; bf16 k and v are exact in tf32, so their lo is 0
+        const bool x_exact = sizeof(T) == 2 && chunk_dim(c, d) < 2 * d;
 #pragma unroll
         for (int p = 0; p < 3; ++p) {
+          if (p == 2 && x_exact) continue;
           const uint32_t xa = xb + (p == 2 ? SC_XB : 0), wa = wb + (p == 1 ? WB : 0);
 #pragma unroll
           for (int ks = 0; ks < SC_KC / 8; ++ks)
@@ -245,7 +249,10 @@ __global__ void __launch_bounds__(SC_THREADS, 1)
 #pragma unroll
         for (int j = 0; j < KVI; ++j) {
           const int it = tid + j * SC_BUILD;
-          split_store(buf, it >> 3, it & 7, to4(cur[j]));
+          if constexpr (sizeof(T) == 2)   // exact in tf32: the head alone (no lo product runs)
+            *reinterpret_cast<float4*>(smf + buf + tile_off(it >> 3, it & 7, SC_M)) = to4(cur[j]);
+          else
+            split_store(buf, it >> 3, it & 7, to4(cur[j]));
         }
       } else {
         const int dim0 = chunk_dim(c, d) - 2 * d;
