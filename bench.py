@@ -350,7 +350,7 @@ def run_kvpop(args):
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for i in range(E):
-        cache.step_host(qh[i], kh[i], vh[i], outh)
+        cache.step_host(qh[i], kh[i], vh[i], outh, stream=stream)
         stream.synchronize()          # the host reads each step's output
     e2e_s = time.perf_counter() - t0
     cache.check()
