@@ -1,6 +1,7 @@
 """Host-side logic of bench.py: multi-rank aggregation (world size 2 over gloo on
-CPU), the algorithmic byte count, sampling of oracle pairs and the committed
-traffic figure."""
+CPU), the algorithmic byte count, sampling of oracle pairs, the committed
+traffic figure, and the reference arm's JSON line (the oracle on host cores), alone
+and under torchrun with two ranks, where rank 0 alone prints it."""
 import os
 import socket
 
@@ -73,3 +74,55 @@ def test_committed_traffic_requires_matching_config():
     assert bench.committed_traffic("ragged") is None
     t = bench.committed_traffic("cr8x")
     assert t is None or t > 1_000_000_000
+
+
+# ---------------------------------------------------------------- the reference arm's JSON line
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+REQUIRED = ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+            "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config")
+
+
+def _json_lines(out):
+    import json
+    return [json.loads(l) for l in out.splitlines() if l.startswith("{")]
+
+
+def _check_reference_line(rec, n_gpus, steps, warmup):
+    for k in REQUIRED:
+        assert k in rec, k
+    assert rec["impl"] == "reference"
+    assert rec["n_gpus"] == n_gpus and rec["steps"] == steps and rec["warmup"] == warmup
+    assert rec["value"] > 0 and rec["unit"] == "tokens/s" and rec["higher_is_better"] is True
+    assert rec["vs_baseline"] is None and rec["config"]["workload"].startswith("tiny")
+    cb = rec["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and isinstance(cb["sample"], str)
+    assert cb["value"] == rec["value"]
+    e = rec["e2e"]
+    assert e["value"] == rec["value"] and e["unit"] == rec["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_reference_arm_prints_one_contract_line():
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "tiny",
+                        "--steps", "2", "--warmup", "3"], cwd=ROOT, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    recs = _json_lines(r.stdout)
+    assert len(recs) == 1
+    _check_reference_line(recs[0], 1, 2, 3)
+
+
+def test_reference_arm_under_torchrun_prints_once_from_rank0():
+    import subprocess
+    import sys
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port()), "bench.py",
+           "--impl", "reference", "--config", "tiny", "--gpus", "2", "--steps", "1", "--warmup", "3"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600,
+                       env=dict(os.environ, OMP_NUM_THREADS="1"))
+    assert r.returncode == 0, r.stderr[-2000:]
+    recs = _json_lines(r.stdout)
+    assert len(recs) == 1
+    _check_reference_line(recs[0], 2, 1, 3)
