@@ -1,5 +1,6 @@
 """Host-only checks of the C ABI: the library loads, exports every declared
-symbol, and rejects bad arguments before touching a GPU."""
+symbol, and rejects bad arguments before touching a GPU; the binding refuses to
+import without the library, and the product package never reaches the oracle."""
 import ctypes
 import os
 import re
@@ -148,3 +149,33 @@ def test_causal_lse_and_future_target_reject_bad_arguments(kv):
     assert ft(*args(G=3)) == bad
     assert ft(*args(lse=P + 2)) == align
     assert ft(*args(tgt=P + 1)) == align
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    """A copy of the binding next to no libkvpop.so must refuse to import (no fallback)."""
+    import importlib.util
+    src = os.path.join(ROOT, "paper_2607_05061_gb300", "kvpop.py")
+    dst = tmp_path / "kvpop.py"
+    dst.write_text(open(src).read())
+    spec = importlib.util.spec_from_file_location("kvpop_nolib", str(dst))
+    mod = importlib.util.module_from_spec(spec)
+    with pytest.raises(ImportError, match="libkvpop.so is missing"):
+        spec.loader.exec_module(mod)
+
+
+def test_product_package_never_reaches_the_oracle():
+    """No file of the product package imports, loads or names the test oracle."""
+    import re
+    pkg = os.path.join(ROOT, "paper_2607_05061_gb300")
+    pat = re.compile(r"\boracle\b")
+    hits = []
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath or "__pycache__" in dirpath:
+            continue
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                path = os.path.join(dirpath, f)
+                for i, line in enumerate(open(path, encoding="utf-8"), 1):
+                    if pat.search(line):
+                        hits.append(f"{os.path.relpath(path, ROOT)}:{i}: {line.strip()}")
+    assert not hits, "\n".join(hits)
