@@ -9,7 +9,7 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
 * Eligible set E(q) = {t | s <= t <= q - w}; the token t_new = q - w has just
   left the protected window (Sec. 3.1, Eq. 4).
 * Delayed scoring: a token is scored only when it leaves the window, with the
-  context gathered meanwhile (Sec. 3.3 "Stateful scorers"; App. E.4).  The
+  context gathered meanwhile (Sec. 3.3, its paragraph on stateful scorers; App. E.4).  The
   scorer is the stateless two-layer MLP of Sec. 3.3 / App. E.2 applied to the
   input [k_u; v_u; qbar_u], where qbar_u averages the D queries u+1..u+D over
   the G query heads that share the KV head, with an exact-erf GELU hidden layer;
@@ -17,9 +17,9 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
   identity hidden layer.
 * Static priority for decay step n = 1: rbar = r - u * log(gamma_h)
   (App. B.3); with log(gamma) = 0 it is the raw score.
-* Running top-k under a fixed budget (Sec. 3.2 "Running top-k sparse
-  attention", App. C.1 mask definition): a newly eligible token enters a free
-  slot while fewer than B slots are used; afterwards it replaces the slot of
+* Running top-k under a fixed budget (Sec. 3.2, App. C.1 mask definition): a
+  newly eligible token enters a free slot while fewer than B slots are used;
+  afterwards it replaces the slot of
   lowest priority (ties -> lowest slot index) iff its priority is strictly
   larger, else it is dropped.  Because priorities are static and E(q) only
   grows, this keeps exactly the running top-k of App. C.1.
