@@ -188,8 +188,11 @@ def test_full_size_gpu_scorer(cuda_device):
         assert np.all(np.abs(got - want) <= 5e-5 * (1.0 + np.abs(want)))
         pos, sc = cache.pair_state(b, h)
         o = set(tr.cache.kept_positions())
+        # end-to-end decisions with each side's own scores: reported, not gated
+        ev = g.evict[:, b, h]
+        same = (ev[:, 0] == np.asarray(tr.slots)) & (ev[:, 1] == np.asarray(tr.evicted))
         print(f"cr8x GPU scorer {(b, h)}: final kept-set agreement "
-              f"{len(o & set(pos)) / len(o):.4f}")
+              f"{len(o & set(pos)) / len(o):.4f}; decode eviction agreement {same.mean():.4f}")
     cache.free()
 
 
