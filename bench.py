@@ -713,6 +713,68 @@ def cpu_prompt_baseline(cfg, over, group, kind):
                        f"per core in parallel: {what}, extrapolated to the whole prompt and group")}
 
 
+def prompt_metric(workload):
+    """(metric, step description) of the prompt / target lines, shared by both arms."""
+    if workload == "prompt":
+        return ("prompt tokens/sec with outputs under the running top-k mask (1 GB300)",
+                "kvpop_prefill_attend: delayed scorer on every prompt token, prompt compression, "
+                "static ranks + running top-k cutoffs, masked causal attention with y and LSE")
+    return ("future-target tokens/sec (transposed attention pass + aggregation, 1 GB300)",
+            "kvpop_future_target with the prompt pass's sparse LSE: log future mass per key "
+            "and query head, max aggregation, count normalisation")
+
+
+def prompt_workload_config(cfg, n):
+    P, H, G, d = cfg.prompt_len, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim
+    return (f"{cfg.name} prompt group: {n} sequences x {P} tokens, {H} KV heads x {G} query heads, "
+            f"d {d}, B {cfg.budget_B}, D {cfg.delay_D}")
+
+
+def run_reference_prompt(args):
+    """The oracle as the reference arm of --workload prompt / target: one (sequence, KV head)
+    pair per step on one core, extrapolated to the whole group (rank 0 only)."""
+    rank, _, world = dist_info()
+    if rank != 0:
+        return
+    from workload import get_config
+    over = {}
+    if args.batch:
+        over["batch"] = args.batch
+    if args.prompt_len:
+        over["prompt_len"] = args.prompt_len
+    cfg = get_config(args.config, **over)
+    if cfg.n_layers != 1 or cfg.ragged:
+        raise SystemExit("--workload prompt/target runs fixed-length single-layer workloads")
+    n = min(args.group, cfg.batch)
+    W, K = args.warmup, args.steps
+    job = _oracle_prompt_job if args.workload == "prompt" else _oracle_target_job
+    nsample = 8 if args.workload == "prompt" else 16       # queries / keys timed per pair
+    times = []
+    for s in range(W + K):
+        b, h = s % n, s % cfg.n_kv_heads
+        t = job((cfg.name, b, h, nsample, over))          # extrapolated to the pair's P
+        if s >= W:
+            times.append(t)
+    pair_s = statistics.mean(times)
+    step_s = n * cfg.n_kv_heads * pair_s
+    value = n * cfg.prompt_len / step_s
+    metric, what = prompt_metric(args.workload)
+    rec = {
+        "metric": metric, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded counter-based generator)",
+        "impl": "reference",
+        "config": {"workload": prompt_workload_config(cfg, n), "step": what},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": (f"each step = one (sequence, KV head) pair of the {n}-sequence "
+                                    f"group on one core ({nsample} evenly spaced "
+                                    f"{'queries' if args.workload == 'prompt' else 'keys'}, "
+                                    f"extrapolated to the prompt), then to the whole group by pairs")},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(rec), flush=True)
+
+
 def run_prompt_bench(args):
     import torch
     rank_, local_rank, world = dist_info()
@@ -829,25 +891,19 @@ def run_prompt_bench(args):
                                             else "target_t5_kernel_traffic.txt"))
     traffic = (committed_traffic(cfg.name, tfile, sequences=n)
                if (cfg.kv_dtype == "bf16" and d == 128 and not over) else None)
+    metric, what = prompt_metric(args.workload)
     if args.workload == "prompt":
-        metric = "prompt tokens/sec with outputs under the running top-k mask (1 GB300)"
         kname = (("prompt_t5_kernel" if d == 128 and not os.environ.get("KVPOP_PROMPT_MMA_SYNC")
                   else "prompt_tc_kernel") if cfg.kv_dtype == "bf16" else "prompt_simt_kernel")
-        what = ("kvpop_prefill_attend: delayed scorer on every prompt token, prompt compression, "
-                "static ranks + running top-k cutoffs, masked causal attention with y and LSE")
     else:
-        metric = "future-target tokens/sec (transposed attention pass + aggregation, 1 GB300)"
         kname = (("target_t5_kernel" if d == 128 and not os.environ.get("KVPOP_TARGET_MMA_SYNC")
                   else "target_tc_kernel") if cfg.kv_dtype == "bf16" else "target_simt_kernel")
-        what = ("kvpop_future_target with the prompt pass's sparse LSE: log future mass per key "
-                "and query head, max aggregation, count normalisation")
     rec = {
         "metric": metric, "value": tokens / (step_ms / 1e3), "unit": "tokens/s", "n_gpus": world,
         "steps": Kn, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": cfg.kv_dtype,
         "data": "synthetic (seeded counter-based generator)",
-        "config": {"workload": f"{cfg.name} prompt group: {n} sequences x {P} tokens, {H} KV heads "
-                               f"x {G} query heads, d {d}, B {cfg.budget_B}, D {cfg.delay_D}",
+        "config": {"workload": prompt_workload_config(cfg, n),
                    "step": what,
                    "l2": f"inputs larger than L2: Q/K/V {(Q.numel() + K.numel() + V.numel()) * 2 / 1e9:.2f} GB",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
@@ -872,7 +928,10 @@ def run_prompt_bench(args):
 def main():
     args = parse_args()
     if args.impl == "reference":
-        run_reference(args)
+        if args.workload == "decode":
+            run_reference(args)
+        else:
+            run_reference_prompt(args)
     elif args.workload != "decode":
         run_prompt_bench(args)
     else:

@@ -102,16 +102,20 @@ def _check_reference_line(rec, n_gpus, steps, warmup):
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
 
 
-def test_reference_arm_prints_one_contract_line():
+@pytest.mark.parametrize("workload", ["decode", "prompt", "target"])
+def test_reference_arm_prints_one_contract_line(workload):
     import subprocess
     import sys
-    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "tiny",
-                        "--steps", "2", "--warmup", "3"], cwd=ROOT, capture_output=True, text=True,
-                       timeout=600)
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload", workload,
+                        "--config", "tiny", "--steps", "2", "--warmup", "3"], cwd=ROOT,
+                       capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
     recs = _json_lines(r.stdout)
     assert len(recs) == 1
     _check_reference_line(recs[0], 1, 2, 3)
+    # the same metric as the GPU arm of that workload
+    want = bench.METRIC if workload == "decode" else bench.prompt_metric(workload)[0]
+    assert recs[0]["metric"] == want
 
 
 def test_reference_arm_under_torchrun_prints_once_from_rank0():
