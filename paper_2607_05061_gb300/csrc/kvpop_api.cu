@@ -88,8 +88,24 @@ kvpop_status dev_alloc(kvpop_cache* c, void** p, size_t bytes) {
     *p = nullptr;
     return from_cuda(e);
   }
-  c->allocs.push_back(*p);
+  try {
+    c->allocs.push_back(*p);
+  } catch (...) {                 // host out of memory: no exception crosses the ABI
+    cudaFree(*p);
+    *p = nullptr;
+    return KVPOP_ERR_OOM;
+  }
   return KVPOP_OK;
+}
+
+// v = n zero bytes; false when the host allocation fails
+bool assign_zero(std::vector<unsigned char>& v, size_t n) {
+  try {
+    v.assign(n, 0);
+  } catch (...) {
+    return false;
+  }
+  return true;
 }
 
 void release(kvpop_cache* c) {
@@ -139,34 +155,37 @@ struct StateBuf {
   void* ptr;
   size_t bytes;
 };
+// The cache's state buffers in a fixed order (the checkpoint format); no allocation.
+struct StateList {
+  StateBuf b[16];
+  int n = 0;
+  void add(void* ptr, size_t bytes) { b[n++] = {ptr, bytes}; }
+  const StateBuf* begin() const { return b; }
+  const StateBuf* end() const { return b + n; }
+};
 
-std::vector<StateBuf> state_buffers(kvpop_cache* c) {
+StateList all_state_buffers(kvpop_cache* c) {
   const Dims& dm = c->dm;
   const size_t pairs = dm.pairs;
-  return {
-      {c->st.slotK, pairs * dm.B * dm.d * c->esz},
-      {c->st.slotV, pairs * dm.B * dm.d * c->esz},
-      {c->st.ringK, pairs * dm.D * dm.d * c->esz},
-      {c->st.ringV, pairs * dm.D * dm.d * c->esz},
-      {c->st.ringQm, pairs * dm.D * dm.d * 4},
-      {c->st.score, pairs * dm.B * 4},
-      {c->st.pos, pairs * dm.B * 4},
-      {c->st.nvalid, pairs * 4},
-      {c->st.len, pairs * 4},
-      {c->st.min_score, pairs * 4},
-      {c->st.min_slot, pairs * 4},
-      {c->st.blk_score, pairs * min_blocks(dm.B) * 4},
-      {c->st.blk_slot, pairs * min_blocks(dm.B) * 4},
-  };
-}
-
-std::vector<StateBuf> all_state_buffers(kvpop_cache* c) {
-  std::vector<StateBuf> v = state_buffers(c);
+  StateList v;
+  v.add(c->st.slotK, pairs * dm.B * dm.d * c->esz);
+  v.add(c->st.slotV, pairs * dm.B * dm.d * c->esz);
+  v.add(c->st.ringK, pairs * dm.D * dm.d * c->esz);
+  v.add(c->st.ringV, pairs * dm.D * dm.d * c->esz);
+  v.add(c->st.ringQm, pairs * dm.D * dm.d * 4);
+  v.add(c->st.score, pairs * dm.B * 4);
+  v.add(c->st.pos, pairs * dm.B * 4);
+  v.add(c->st.nvalid, pairs * 4);
+  v.add(c->st.len, pairs * 4);
+  v.add(c->st.min_score, pairs * 4);
+  v.add(c->st.min_slot, pairs * 4);
+  v.add(c->st.blk_score, pairs * min_blocks(dm.B) * 4);
+  v.add(c->st.blk_slot, pairs * min_blocks(dm.B) * 4);
   if (c->mlstm) {
-    const size_t pairs = c->dm.pairs, d = c->dm.d;
-    v.push_back({c->md.C, pairs * d * (d / 2) * 4});
-    v.push_back({c->md.z, pairs * d * 4});
-    v.push_back({c->md.m, pairs * 4});
+    const size_t d = dm.d;
+    v.add(c->md.C, pairs * d * (d / 2) * 4);
+    v.add(c->md.z, pairs * d * 4);
+    v.add(c->md.m, pairs * 4);
   }
   return v;
 }
@@ -284,8 +303,8 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
   }
   if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * dm.G * d * 4); c->stage_out = (float*)p; }
   if (s == KVPOP_OK && c->use_tc) {
-    c->tc_maps.assign(tc_maps_size() + 64, 0);
-    s = from_cuda(NOTE(tc_make_maps(c->st, dm, tc_map_ptr(c))));
+    s = assign_zero(c->tc_maps, tc_maps_size() + 64) ? from_cuda(NOTE(tc_make_maps(c->st, dm, tc_map_ptr(c))))
+                                                     : KVPOP_ERR_OOM;
   }
   if (s == KVPOP_OK) s = from_cuda(NOTE(prepare_ingest(dm)));
   const size_t hh = d / 2, NCm = mlstm_nc(dm.d);
@@ -316,7 +335,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
   if (s == KVPOP_OK && c->use_tf32) {
     s = dev_alloc(c, &p, 2 * H * dm.F * I * 4);
     c->w1t = (float*)p;
-    c->sc_maps.assign(score_tf32_maps_size() + 64, 0);
+    if (s == KVPOP_OK && !assign_zero(c->sc_maps, score_tf32_maps_size() + 64)) s = KVPOP_ERR_OOM;
   }
   if (s == KVPOP_OK) {
     float* W1 = w;
@@ -362,7 +381,11 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
       if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(md.a, ms->a, H * hh * 4, cudaMemcpyDefault, stream));
       if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(md.C, 0, pairs * d * hh * 4, stream));
       if (e == cudaSuccess) e = NOTE(cudaMemsetAsync(md.z, 0, pairs * d * 4, stream));
-      minus_inf.assign(pairs, -INFINITY);
+      try {
+        minus_inf.assign(pairs, -INFINITY);
+      } catch (...) {
+        if (e == cudaSuccess) e = cudaErrorMemoryAllocation;
+      }
       if (e == cudaSuccess)
         e = NOTE(cudaMemcpyAsync(md.m, minus_inf.data(), pairs * 4, cudaMemcpyHostToDevice, stream));
     }
@@ -784,7 +807,12 @@ kvpop_status kvpop_get_lengths(kvpop_cache* c, int32_t* len_host, cudaStream_t s
   kvpop_status s = usable(c);
   if (s != KVPOP_OK) return s;
   if (!len_host) return KVPOP_ERR_INVALID_ARG;
-  std::vector<int32_t> all((size_t)c->dm.pairs);
+  std::vector<int32_t> all;
+  try {
+    all.resize((size_t)c->dm.pairs);
+  } catch (...) {
+    return KVPOP_ERR_OOM;
+  }
   cudaError_t e = NOTE(cudaMemcpyAsync(all.data(), c->st.len, all.size() * 4, cudaMemcpyDeviceToHost, stream));
   if (e == cudaSuccess) e = NOTE(cudaStreamSynchronize(stream));
   if (e != cudaSuccess) return poison_on(c, e);
