@@ -157,9 +157,12 @@ struct StateBuf {
 };
 // The cache's state buffers in a fixed order (the checkpoint format); no allocation.
 struct StateList {
-  StateBuf b[16];
+  static constexpr int kMax = 24;     // 16 in use (13 + 3 for the mLSTM state)
+  StateBuf b[kMax];
   int n = 0;
-  void add(void* ptr, size_t bytes) { b[n++] = {ptr, bytes}; }
+  void add(void* ptr, size_t bytes) {
+    if (n < kMax) b[n++] = {ptr, bytes};
+  }
   const StateBuf* begin() const { return b; }
   const StateBuf* end() const { return b + n; }
 };
