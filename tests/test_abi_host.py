@@ -53,7 +53,8 @@ def good_config(kv, **kw):
 @pytest.mark.parametrize("field,value", [
     ("batch", 0), ("n_kv_heads", 0), ("q_per_kv", 3), ("q_per_kv", 8), ("head_dim", 96),
     ("budget_B", 0), ("delay_D", 0), ("n_sink", -1), ("n_sink", 8), ("scorer_hidden", 0),
-    ("scorer_hidden", 2048), ("kv_dtype", 7), ("batch", 100000)])
+    ("scorer_hidden", 2048), ("kv_dtype", 7), ("batch", 100000),
+    ("batch", 6145)])                # 12290 pairs: one past the largest accepted 12288
 def test_init_rejects_bad_config(kv, field, value):
     cfg = good_config(kv, **{field: value})
     buf = (ctypes.c_float * 16)()
