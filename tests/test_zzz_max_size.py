@@ -20,7 +20,7 @@ MAX_PAIRS = 12288
 
 def test_largest_accepted_pair_count(cuda_device):
     cfg = get_config("q4b", batch=MAX_PAIRS // 8, prompt_len=24, budget_B=16, delay_D=4,
-                     scorer_hidden=32, decode_steps=6)
+                     decode_steps=6)
     assert cfg.batch * cfg.n_kv_heads == MAX_PAIRS
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
