@@ -9,8 +9,9 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
 * Eligible set E(q) = {t | s <= t <= q - w}; the token t_new = q - w has just
   left the protected window (Sec. 3.1, Eq. 4).
 * Delayed scoring: a token is scored only when it leaves the window, with the
-  context gathered meanwhile (Sec. 3.3, its paragraph on stateful scorers; App. E.4).  The
-  scorer is the stateless two-layer MLP of Sec. 3.3 / App. E.2 applied to the
+  context gathered meanwhile (Sec. 3.3, its paragraph on stateful scorers;
+  App. E.4).  The scorer is the stateless two-layer MLP of Sec. 3.3 / App. E.2
+  applied to the
   input [k_u; v_u; qbar_u], where qbar_u averages the D queries u+1..u+D over
   the G query heads that share the KV head, with an exact-erf GELU hidden layer;
   or the paper's plain variant on [k_u; v_u] (W1 with 2d rows), with a SiLU or
@@ -19,9 +20,8 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
   (App. B.3); with log(gamma) = 0 it is the raw score.
 * Running top-k under a fixed budget (Sec. 3.2, App. C.1 mask definition): a
   newly eligible token enters a free slot while fewer than B slots are used;
-  afterwards it replaces the slot of
-  lowest priority (ties -> lowest slot index) iff its priority is strictly
-  larger, else it is dropped.  Because priorities are static and E(q) only
+  afterwards it replaces the slot of lowest priority (ties -> lowest slot
+  index) iff its priority is strictly larger, else it is dropped.  Because priorities are static and E(q) only
   grows, this keeps exactly the running top-k of App. C.1.
 * Decode attends over the compact cache only: slots plus the w pending tokens
   (App. C, first paragraph), softmax(q k^T / sqrt(d)) v per query head.
@@ -34,8 +34,9 @@ order as the CUDA path, because that value decides an integer (the kept slot).
 Parity status: the attention, window and eviction logic are pinned by tests
 (dense-attention reduction, brute-force top-k subsets, the App. C.1 mask
 recomputed from scratch).  The scorer's exact form ([k; v; mean of the next D
-queries], GELU, F hidden units) is a workload choice the paper does not print;
-it is pinned only at hand-set weights and closed-form GELU values.
+queries], GELU, F hidden units) is a workload choice the paper does not print:
+parity unpinned for that form against the paper; the oracle's scorer is pinned
+only at hand-set weights and closed-form GELU values.
 """
 from __future__ import annotations
 
