@@ -11,9 +11,9 @@ w = D, long-range top-k, budget slots B = s + k; the window is held apart):
 * Delayed scoring: a token is scored only when it leaves the window, with the
   context gathered meanwhile (Sec. 3.3, its paragraph on stateful scorers;
   App. E.4).  The scorer is the stateless two-layer MLP of Sec. 3.3 / App. E.2
-  applied to the
-  input [k_u; v_u; qbar_u], where qbar_u averages the D queries u+1..u+D over
-  the G query heads that share the KV head, with an exact-erf GELU hidden layer;
+  applied to the input [k_u; v_u; qbar_u], where qbar_u averages the D queries
+  u+1..u+D over the G query heads that share the KV head, with an exact-erf
+  GELU hidden layer;
   or the paper's plain variant on [k_u; v_u] (W1 with 2d rows), with a SiLU or
   identity hidden layer.
 * Static priority for decay step n = 1: rbar = r - u * log(gamma_h)
