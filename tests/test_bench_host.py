@@ -1,7 +1,9 @@
 """Host-side logic of bench.py: multi-rank aggregation (world size 2 over gloo on
 CPU), the algorithmic byte count, sampling of oracle pairs, the committed
-traffic figure, and the reference arm's JSON line (the oracle on host cores), alone
-and under torchrun with two ranks, where rank 0 alone prints it."""
+traffic figure, the prompt and target flop counts behind their roofline (against the
+oracle's mask and a pair-by-pair count), and the reference arm's JSON line (the
+oracle on host cores), alone and under torchrun with two ranks, where rank 0 alone
+prints it."""
 import os
 import socket
 
@@ -130,3 +132,28 @@ def test_reference_arm_under_torchrun_prints_once_from_rank0():
     recs = _json_lines(r.stdout)
     assert len(recs) == 1
     _check_reference_line(recs[0], 2, 1, 3)
+
+
+# ---------------------------------------------------------------- roofline arithmetic of the prompt paths
+@pytest.mark.parametrize("P,B,D,s", [(60, 16, 4, 0), (97, 24, 7, 3), (10, 16, 4, 2)])
+def test_prompt_flops_count_the_oracle_mask(P, B, D, s):
+    """4 d G per retained (query, key) of the running top-k mask built by the oracle."""
+    import numpy as np
+    from oracle import running_topk as rt
+    cfg = get_config("q4b", batch=1, prompt_len=P, budget_B=B, delay_D=D, n_sink=s)
+    raw = np.random.default_rng(P).standard_normal(P).astype(np.float32)
+    prio = rt.prompt_priorities(raw, P, D, 0.0)
+    rank = rt.static_ranks(prio)
+    tau = rt.fenwick_cutoffs(rank, s, D, B - s)
+    kept = sum(int(rt.mask_row(q, rank, tau, s, D).sum()) for q in range(P))
+    want = 4.0 * cfg.head_dim * cfg.q_per_kv * cfg.n_kv_heads * kept
+    assert bench.prompt_attention_flops(cfg, [P]) == want
+
+
+@pytest.mark.parametrize("P,D", [(50, 4), (7, 16), (33, 1)])
+def test_target_flops_count_key_query_pairs(P, D):
+    """2 d G per (key t, query d) with t + w <= d < P, counted one by one."""
+    cfg = get_config("q4b", batch=1, prompt_len=P, delay_D=D)
+    pairs = sum(1 for t in range(P) for d in range(P) if d >= t + D)
+    want = 2.0 * cfg.head_dim * cfg.q_per_kv * cfg.n_kv_heads * pairs
+    assert bench.target_flops(cfg, [P]) == want
