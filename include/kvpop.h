@@ -2,9 +2,9 @@
  * kvpop.h -- C ABI of the KVpop decode hot path on one GB300 (sm_103a).
  *
  * KVpop ("KV cache compression with predictive online pruning") keeps, per KV
- * head, s sink tokens, a protected window of the w most recent tokens and a
- * long-range top-k set chosen by a learned scorer (Sec. 3, Eq. 1).  Per decode
- * step this library
+ * head, the first s tokens (sinks), the last w tokens, which are never
+ * evicted, and a long-range top-k set chosen by a learned scorer (Sec. 3,
+ * Eq. 1).  Per decode step this library
  *   1. ingests the new token's q/k/v into the window,
  *   2. scores the token u = p - w that has just left the window with the
  *      delayed scorer (Sec. 3.3, App. E.4): a two-layer MLP on
@@ -112,8 +112,10 @@ typedef struct kvpop_cache kvpop_cache;   /* opaque, library-owned device state 
 /* Human-readable name of a status (static string, never NULL). */
 const char* kvpop_status_string(kvpop_status s);
 
-/* Create an empty cache (length 0 for every sequence) on the current device.
- * Allocates the slot store [b][H][B][d] for K and V, the window rings
+/* Create an empty cache (length 0 for every sequence) on the current device:
+ * the per-KV-head state the method keeps under its fixed budget (Sec. 3,
+ * Eq. 1: s sink + k long-range slots, here B = s + k, and the window of w = D
+ * tokens held apart) plus the stateless scorer of Sec. 3.3.  Allocates the slot store [b][H][B][d] for K and V, the window rings
  * [b][H][D][d], per-slot score/position arrays and the attention workspace.
  * Synchronises `stream` before returning.  *out is NULL on failure. */
 kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* scorer,
@@ -126,7 +128,8 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* score
 kvpop_status kvpop_init_cache_mlstm(const kvpop_config* cfg, const kvpop_mlstm_scorer* scorer,
                                     cudaStream_t stream, kvpop_cache** out);
 
-/* Release the cache and all its device memory.  kvpop_free(NULL) is KVPOP_OK.
+/* Release the cache and all its device memory (resource management; the paper
+ * has no counterpart).  kvpop_free(NULL) is KVPOP_OK.
  * Synchronises the device work of the cache first. */
 kvpop_status kvpop_free(kvpop_cache* cache);
 
@@ -141,7 +144,12 @@ kvpop_status kvpop_free(kvpop_cache* cache);
  *   score_override_dev  [n_seq][H][Pmax] fp32 raw scores used instead of the
  *                        scorer (entry u), or NULL
  * Uses a stream-ordered temporary of n_seq*H*Pmax*4 bytes and synchronises
- * `stream` before returning (the host length array may be reused at once). */
+ * `stream` before returning (the host length array may be reused at once).
+ * The lengths are host values and the batch may come in chunks of sequences
+ * because a whole batch's prompts need not fit in device memory at once (128
+ * ragged prompts of up to 65536 tokens are about 35 GB of bf16 Q/K/V); the
+ * temporary is sized from the chunk, and the call returns only once the host
+ * length array is no longer read. */
 kvpop_status kvpop_prefill_compress(kvpop_cache* cache, const void* Q_dev, const void* K_dev,
                                     const void* V_dev, const int32_t* prompt_len_host,
                                     int32_t first_seq, int32_t n_seq, int32_t Pmax,
@@ -262,7 +270,10 @@ kvpop_status kvpop_future_target(const void* Q_dev, const void* K_dev, const flo
                                  cudaStream_t stream);
 
 /* Decode steps 1-4 for every sequence: ingest the token at position p = len,
- * score u = p - D (if p >= D), keep or drop it, scatter it, push p.
+ * score u = p - D (if p >= D; the token that has just become eligible, Sec. 3.1
+ * Eq. 4) with the delayed scorer (Sec. 3.3, App. E.4), keep or drop it under the
+ * budget (Sec. 3.2 running top-k, App. C.1 mask, App. B.3 static priority),
+ * scatter it, push p.
  *   q_dev [b][H*G][d], k_dev / v_dev [b][H][d]
  *   score_override_dev [b][H] fp32 raw scores used instead of the scorer, or NULL
  *   evict_info_dev [b][H][2] int32 out: (slot u went to or -1, evicted position
@@ -274,8 +285,9 @@ kvpop_status kvpop_decode_ingest(kvpop_cache* cache, const void* q_dev, const vo
                                  int32_t* evict_info_dev, float* score_out_dev,
                                  cudaStream_t stream);
 
-/* Decode step 5: out_g = softmax(q_g K_S^T / sqrt(d)) V_S for every query head,
- * where S = kept slots plus window entries of its KV head.  Split-K over a
+/* Decode step 5 (App. C, first paragraph: decode attends over the compact cache
+ * only): out_g = softmax(q_g K_S^T / sqrt(d)) V_S for every query head, where
+ * S = kept slots plus window entries of its KV head.  Split-K over a
  * persistent grid with token-balanced ranges.
  *   q_dev [b][H*G][d] (same as ingest)   out_dev [b][H*G][d] fp32 */
 kvpop_status kvpop_decode_attend(kvpop_cache* cache, const void* q_dev, float* out_dev,

@@ -15,7 +15,7 @@ and long-range budget k (the build's B = s + k, D = w):
   the mask definition disagree: Algorithm 2 leaves tau_q = -1 while fewer than
   k tokens are eligible, which, read literally, keeps none of them; the mask
   definition keeps the top k of E(q), i.e. all of E(q) when |E(q)| < k, and
-  the budget binds only once the sequence is longer than s + w + k.  So here
+  the budget starts to evict only when more than s + w + k tokens exist.  So here
   tau_q = FindByPrefixCount(T, min(k, |E(q)|)), and -1 only when E(q) is empty.
 * mask (Eq. in App. C.1): M[q, t] = t < s  or  q - t < w  or
   (s <= t <= q - w and rank(t) <= tau_q), for t <= q.
