@@ -104,6 +104,49 @@ def kv_stream_bytes(cfg, lengths, step: int) -> int:
     return tot * cfg.n_kv_heads * 2 * cfg.head_dim * cfg.esz
 
 
+L2_BYTES = 129e6           # GB300 L2 (126 MiB)
+FLUSH_BYTES = 512 << 20    # written between timed steps whose inputs fit in twice the L2
+ATTN_POST_LAUNCHES = 32    # event-timed attention launches after a short timed region
+
+
+def flushes_l2(bytes_per_step: float) -> bool:
+    """Whether a step's inputs are too small to push the last step's data out of L2."""
+    return bytes_per_step < 2 * L2_BYTES
+
+
+def decode_dtype(cfg) -> str:
+    """The arithmetic of the decode path: bf16 K/V products on tensor cores with fp32
+    accumulation (P rounded to bf16 for the PV product), or fp32 throughout."""
+    return "bf16 (fp32 accumulate)" if cfg.kv_dtype == "bf16" else "f32"
+
+
+def scorer_description(cfg, scorer: str) -> str:
+    if scorer == "mlstm":
+        return (f"stateful delayed mLSTM (Hedgehog, C {cfg.head_dim}x{cfg.head_dim // 2} per "
+                f"head) fp32")
+    return f"MLP {cfg.scorer_in}->{cfg.scorer_hidden} GELU->1 fp32"
+
+
+def decode_config(cfg, scorer: str, bytes_per_step: float, world: int) -> dict:
+    """The `config` object of the decode line; both arms print the same one."""
+    if flushes_l2(bytes_per_step):
+        l2 = (f"inputs smaller than twice L2 ({bytes_per_step / 1e9:.3f} GB K/V read per step): "
+              f"a {FLUSH_BYTES >> 20} MiB buffer is written before every timed step, and each "
+              f"step is timed on its own with CUDA events, the flush outside them")
+    else:
+        l2 = f"inputs larger than L2: {bytes_per_step / 1e9:.3f} GB K/V read per step"
+    return {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
+            "kv_heads": cfg.n_kv_heads, "q_per_kv": cfg.q_per_kv, "head_dim": cfg.head_dim,
+            "prompt_len": "ragged U[%d,%d]" % cfg.ragged if cfg.ragged else cfg.prompt_len,
+            "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype,
+            "scorer": scorer_description(cfg, scorer), "l2": l2,
+            "parallelism": "replicas" if world > 1 else "single GPU"}
+
+
+def mean_stream_bytes(cfg, lengths, step0: int, n: int) -> float:
+    return statistics.mean(kv_stream_bytes(cfg, lengths, step0 + i) for i in range(n))
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -192,7 +235,10 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ oracle (CPU) legs
 def _oracle_pair_job(args):
-    """Prefill one (sequence, KV head) in the oracle (untimed), then time n decode steps."""
+    """Prefill one (sequence, KV head) in the oracle (untimed), then time n decode steps.
+
+    Returns (seconds, kept positions after the prefill, per-step (slot, evicted
+    position) decisions) -- the decisions feed the eviction-agreement report."""
     cfg_name, b, h, n_steps, scorer = args
     import torch
     torch.set_num_threads(1)
@@ -204,16 +250,19 @@ def _oracle_pair_job(args):
         cache = prefill_pair_mlstm(cfg, gen.mlstm_weights(cfg), b, h, L[b])
     else:
         cache = prefill_pair(cfg, gen.scorer_weights(cfg), b, h, L[b])
+    kept = cache.kept_positions()
     G = cfg.q_per_kv
     q, k, v = gen.decode_inputs(cfg, [L[b]], 0, n_steps, b0=b)
     q = q[:, 0, h * G:(h + 1) * G].double().numpy()
     k = k[:, 0, h].double().numpy()
     v = v[:, 0, h].double().numpy()
+    decisions = []
     t0 = time.perf_counter()
     for j in range(n_steps):
-        cache.append(q[j], k[j], v[j])
+        slot, ev, _ = cache.append(q[j], k[j], v[j])
         cache.attend(q[j])
-    return time.perf_counter() - t0
+        decisions.append((int(slot), int(ev)))
+    return time.perf_counter() - t0, kept, decisions
 
 
 def sample_pairs(cfg, n):
@@ -222,23 +271,57 @@ def sample_pairs(cfg, n):
     return [(i // cfg.n_kv_heads, i % cfg.n_kv_heads) for i in idx]
 
 
+def baseline_pairs(cfg):
+    """The (sequence, KV head) pairs the CPU baseline runs: one per host core, at most 16."""
+    return sample_pairs(cfg, max(1, min(os.cpu_count() or 1, 16)))
+
+
 def cpu_baseline(cfg, n_steps: int, scorer: str = "mlp"):
-    """fp64 oracle decode throughput on this host's cores (spawned pool, one pair per core)."""
+    """fp64 oracle decode throughput on this host's cores (spawned pool, one pair per core).
+
+    Returns (the cpu_baseline object, per-pair (kept positions, decisions))."""
     import multiprocessing as mp
-    cores = max(1, min(os.cpu_count() or 1, 16))
-    pairs = sample_pairs(cfg, cores)
+    pairs = baseline_pairs(cfg)
     for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         os.environ[var] = "1"
     ctx = mp.get_context("spawn")
     with ctx.Pool(len(pairs)) as pool:
-        times = pool.map(_oracle_pair_job, [(cfg.name, b, h, n_steps, scorer) for b, h in pairs])
+        res = pool.map(_oracle_pair_job, [(cfg.name, b, h, n_steps, scorer) for b, h in pairs])
+    times = [r[0] for r in res]
     per_pair_step = statistics.mean(times) / n_steps            # seconds per (pair, step)
     step_time = cfg.batch * cfg.n_kv_heads * per_pair_step / len(pairs)
-    return {"value": cfg.batch / step_time, "unit": "tokens/s", "cores": len(pairs), "kind": "oracle",
-            "sample": (f"{len(pairs)} of {cfg.batch * cfg.n_kv_heads} (sequence, KV head) pairs, "
-                       f"{n_steps} decode steps each after an untimed oracle prefill, one pair per "
-                       f"core in parallel; whole-batch step time extrapolated as pairs/cores x "
-                       f"mean pair-step time")}
+    rec = {"value": cfg.batch / step_time, "unit": "tokens/s", "cores": len(pairs), "kind": "oracle",
+           "sample": (f"{len(pairs)} of {cfg.batch * cfg.n_kv_heads} (sequence, KV head) pairs, "
+                      f"{n_steps} decode steps each after an untimed oracle prefill, one pair per "
+                      f"core in parallel; whole-batch step time extrapolated as pairs/cores x "
+                      f"mean pair-step time")}
+    return rec, {pr: (r[1], r[2]) for pr, r in zip(pairs, res)}
+
+
+def agreement(gpu_kept: dict, gpu_decisions, oracle: dict) -> dict:
+    """End-to-end eviction agreement, each side with its own scores.
+
+    ``gpu_decisions[j][b][h]`` = (slot, evicted position) at decode step j;
+    ``oracle[(b, h)]`` = (kept positions after prefill, per-step decisions)."""
+    n = eq = kept_eq = 0
+    first = None
+    for (b, h), (kept, dec) in sorted(oracle.items()):
+        kept_eq += int(sorted(gpu_kept[(b, h)]) == list(kept))
+        for j, d in enumerate(dec):
+            g = tuple(int(x) for x in gpu_decisions[j][b][h])
+            n += 1
+            if g == tuple(d):
+                eq += 1
+            elif first is None:
+                first = {"pair": [b, h], "step": j, "gpu": list(g), "oracle": list(d)}
+    return {"decode_decisions_equal": eq / n if n else None, "decisions": n,
+            "prefill_kept_sets_equal": kept_eq / len(oracle) if oracle else None,
+            "pairs": len(oracle), "steps": len(next(iter(oracle.values()))[1]) if oracle else 0,
+            "first_mismatch": first,
+            "how": ("each side scores with its own arithmetic (CUDA fp32 kernels; the fp64 oracle "
+                    "rounded to fp32) from the same seeded prompt; a decision is the (slot, evicted "
+                    "position) of one (sequence, KV head) at one decode step; kept sets compared "
+                    "after the prompt compression")}
 
 
 # ------------------------------------------------------------------ GPU arm
@@ -267,33 +350,38 @@ def run_kvpop(args):
         cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
                                  cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, n_sink=cfg.n_sink,
                                  mlstm=gen.mlstm_weights(cfg))
-        scorer_desc = (f"stateful delayed mLSTM (Hedgehog, C {cfg.head_dim}x{cfg.head_dim // 2} per "
-                       f"head) fp32")
     else:
         W1, b1, w2, b2, lg = gen.scorer_weights(cfg)
         cache = kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
                                  cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, W1, b1, w2, b2,
                                  n_sink=cfg.n_sink)
-        scorer_desc = f"MLP {cfg.scorer_in}->{cfg.scorer_hidden} GELU->1 fp32"
-    # prefill (untimed), a few sequences at a time to bound the prompt buffers
-    t_prefill = 0.0
-    group = 8
-    for b0 in range(0, cfg.batch, group):
-        nb = min(group, cfg.batch - b0)
-        Lg = L[b0:b0 + nb]
-        Pm = max(Lg)
-        Q = gen.q_tokens(cfg, b0, nb, 0, Pm, device=dev)
-        K = gen.kv_tokens(cfg, "k", b0, nb, 0, Pm, device=dev)
-        V = gen.kv_tokens(cfg, "v", b0, nb, 0, Pm, device=dev)
-        torch.cuda.synchronize()
-        tp = time.perf_counter()
-        cache.prefill(Q, K, V, Lg, first_seq=b0)
-        t_prefill += time.perf_counter() - tp
-        del Q, K, V
-    torch.cuda.synchronize()
 
+    def prefill_all():
+        """Prompt compression of the whole batch, a few sequences at a time (bounded buffers)."""
+        t = 0.0
+        group = 8
+        for b0 in range(0, cfg.batch, group):
+            nb = min(group, cfg.batch - b0)
+            Lg = L[b0:b0 + nb]
+            Pm = max(Lg)
+            Q = gen.q_tokens(cfg, b0, nb, 0, Pm, device=dev)
+            K = gen.kv_tokens(cfg, "k", b0, nb, 0, Pm, device=dev)
+            V = gen.kv_tokens(cfg, "v", b0, nb, 0, Pm, device=dev)
+            torch.cuda.synchronize()
+            tp = time.perf_counter()
+            cache.prefill(Q, K, V, Lg, first_seq=b0)
+            t += time.perf_counter() - tp
+            del Q, K, V
+        torch.cuda.synchronize()
+        return t
+
+    t_prefill = prefill_all()
     W, K = args.warmup, args.steps
-    q, k, v = gen.decode_inputs(cfg, L, 0, W + K, device=dev)
+    bytes_per_launch = mean_stream_bytes(cfg, L, W, K)
+    flush = flushes_l2(bytes_per_launch)
+    flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev) if flush else None
+    post = ATTN_POST_LAUNCHES if (K < 64 or flush) else 0
+    q, k, v = gen.decode_inputs(cfg, L, 0, W + K + post, device=dev)
     out = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     for j in range(W):
@@ -301,15 +389,19 @@ def run_kvpop(args):
         cache.attend(q[j], out)
     torch.cuda.synchronize()
 
-    # The attention kernel's own duration is sampled with events around it on every
-    # ATTN_SAMPLE-th step; events between the ingest and the attention would stop the
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    # The attention kernel's own duration: with a long timed region, events around it on
+    # every ATTN_SAMPLE-th step (events between the ingest and the attention stop the
     # attention from launching as a programmatic dependent of the ingest, so the other
-    # steps run without them.
-    samples = list(range(0, K, ATTN_SAMPLE))
-    ev_s = {i: torch.cuda.Event(enable_timing=True) for i in samples}
-    ev_e = {i: torch.cuda.Event(enable_timing=True) for i in samples}
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
+    # steps run without them); with a short one, or with L2 flushes, in a loop of
+    # ATTN_POST_LAUNCHES steps after it with events around each attention.
+    samples = [] if post else list(range(0, K, ATTN_SAMPLE))
+    ev_s = {i: ev() for i in samples}
+    ev_e = {i: ev() for i in samples}
+    step_ev = [(ev(), ev()) for _ in range(K)] if flush else []
+    t_start, t_end = ev(), ev()
     clocks = ClockSampler(local_rank)
     clocks.start()
     if world > 1:
@@ -318,6 +410,9 @@ def run_kvpop(args):
     t_start.record(stream)
     for i in range(K):
         j = W + i
+        if flush:
+            flush_buf.fill_(float(i))
+            step_ev[i][0].record(stream)
         cache.ingest(q[j], k[j], v[j])
         if i in ev_s:
             ev_s[i].record(stream)
@@ -325,18 +420,46 @@ def run_kvpop(args):
             ev_e[i].record(stream)
         else:
             cache.attend(q[j], out)
+        if flush:
+            step_ev[i][1].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
     cache.check()
-    step_ms_local = t_start.elapsed_time(t_end) / K
-    attn_ms = statistics.mean(ev_s[i].elapsed_time(ev_e[i]) for i in samples)
+    if flush:
+        step_ms_local = statistics.mean(a.elapsed_time(b) for a, b in step_ev)
+    else:
+        step_ms_local = t_start.elapsed_time(t_end) / K
+    attn_pairs = []
+    if post:
+        for i in range(post):
+            j = W + K + i
+            cache.ingest(q[j], k[j], v[j])
+            if flush:
+                flush_buf.fill_(float(i))
+            a, b = ev(), ev()
+            a.record(stream)
+            cache.attend(q[j], out)
+            b.record(stream)
+            attn_pairs.append((a, b))
+        torch.cuda.synchronize()
+        attn_ms = statistics.mean(a.elapsed_time(b) for a, b in attn_pairs)
+        attn_bytes = mean_stream_bytes(cfg, L, W + K, post)
+        attn_how = (f"CUDA events around the attention in {post} decode steps after the timed "
+                    f"region (the ingest between them untimed" +
+                    (", L2 flushed before each)" if flush else ")"))
+    else:
+        attn_ms = statistics.mean(ev_s[i].elapsed_time(ev_e[i]) for i in samples)
+        attn_bytes = statistics.mean(kv_stream_bytes(cfg, L, W + i) for i in samples)
+        attn_how = (f"CUDA events around the attention on {len(samples)} of the {K} timed steps "
+                    f"(every {ATTN_SAMPLE}th)")
 
     # end to end through the C ABI on host buffers (pinned), copies inside the timed region
     E = max(1, args.e2e_steps)
-    qa, ka, va = gen.decode_inputs(cfg, L, W + K, E, device="cpu")
+    s0 = W + K + post
+    qa, ka, va = gen.decode_inputs(cfg, L, s0, E, device="cpu")
     # each step's q, k, v back to back in one pinned buffer (one host-to-device copy)
     qb, kb = qa[0].numel() * qa.element_size(), ka[0].numel() * ka.element_size()
     packed = torch.empty((E, qb + 2 * kb), dtype=torch.uint8).pin_memory()
@@ -348,33 +471,53 @@ def run_kvpop(args):
             lst.append(view)
     outh = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32).pin_memory()
     torch.cuda.synchronize()
+    e2e_s = 0.0
     t0 = time.perf_counter()
     for i in range(E):
+        if flush:                     # flush, wait, then time the step alone
+            flush_buf.fill_(float(i))
+            stream.synchronize()
+            t0 = time.perf_counter()
         cache.step_host(qh[i], kh[i], vh[i], outh, stream=stream)
         stream.synchronize()          # the host reads each step's output
-    e2e_s = time.perf_counter() - t0
+        if flush:
+            e2e_s += time.perf_counter() - t0
+    if not flush:
+        e2e_s = time.perf_counter() - t0
     cache.check()
     h2d = qb + 2 * kb
     d2h = outh.numel() * 4
+
+    # eviction agreement: the same prompts again, then the first decode steps with every
+    # (slot, evicted position) recorded, for comparison with the oracle's own decisions
+    agree_pairs = baseline_pairs(cfg) if (rank == 0 and not args.no_cpu_baseline) else []
+    gpu_kept, gpu_dec = {}, None
+    if agree_pairs:
+        prefill_all()
+        for b_, h_ in agree_pairs:
+            pos, _ = cache.pair_state(b_, h_)
+            gpu_kept[(b_, h_)] = [int(t) for t in pos]
+        n_ag = args.cpu_steps
+        qg, kg, vg = gen.decode_inputs(cfg, L, 0, n_ag, device=dev)
+        eig = torch.empty((n_ag, cfg.batch, cfg.n_kv_heads, 2), dtype=torch.int32, device=dev)
+        for j in range(n_ag):
+            cache.ingest(qg[j], kg[j], vg[j], evict_info=eig[j])
+        gpu_dec = eig.cpu().numpy()
+        cache.check()
+        del qg, kg, vg
 
     step_ms, _ = reduce_max_sum(step_ms_local, 0.0, world, dev)
     e2e_max, _ = reduce_max_sum(e2e_s / E * 1e3, 0.0, world, dev)
     tokens_per_step = cfg.batch * world
     value = tokens_per_step / (step_ms / 1e3)
-    bytes_per_launch = statistics.mean(kv_stream_bytes(cfg, L, W + i) for i in range(K))
-    achieved = bytes_per_launch / (attn_ms / 1e3) / 1e9
+    achieved = attn_bytes / (attn_ms / 1e3) / 1e9
     peak, peak_src = measured_peaks()
     rec = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded counter-based generator)",
-        "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
-                   "kv_heads": cfg.n_kv_heads, "q_per_kv": cfg.q_per_kv, "head_dim": cfg.head_dim,
-                   "prompt_len": "ragged U[%d,%d]" % cfg.ragged if cfg.ragged else cfg.prompt_len,
-                   "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype,
-                   "scorer": scorer_desc,
-                   "l2": f"inputs larger than L2: {bytes_per_launch / 1e9:.3f} GB K/V read per step",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "vs_baseline": None, "dtype": decode_dtype(cfg),
+        "data": "synthetic (seeded counter-based generator)",
+        "config": decode_config(cfg, args.scorer, bytes_per_launch, world),
         "steps_per_s": 1e3 / step_ms,
         "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
         "prefill_s": t_prefill,
@@ -383,21 +526,23 @@ def run_kvpop(args):
                      "achieved": achieved, "peak": peak,
                      "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
-                     "frac_of_8tbs_nominal": achieved / 8000.0, "traffic": committed_traffic(cfg.name),
-                     "algorithmic_bytes_per_launch": bytes_per_launch, "ms_per_launch": attn_ms,
-                     "ms_per_launch_how": f"CUDA events around the attention on {len(samples)} of the "
-                                          f"{K} timed steps (every {ATTN_SAMPLE}th)"},
+                     "frac_of_8tbs_nominal": achieved / 8000.0,
+                     "traffic": None if over else committed_traffic(cfg.name),
+                     "algorithmic_bytes_per_launch": attn_bytes, "ms_per_launch": attn_ms,
+                     "ms_per_launch_how": attn_how},
         "e2e": {"value": tokens_per_step / (e2e_max / 1e3), "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": E,
                 "how": "kvpop_decode_step_host on pinned host buffers (q|k|v packed: one copy in; "
-                       "the attention writes out into pinned host memory), stream sync every step"},
+                       "the attention writes out into pinned host memory), stream sync every step"
+                       + ("; L2 flushed before each step, outside its timing" if flush else "")},
         "gpu_launches": 2 * K,
         "clocks": clk,
     }
     cache.free()
     del q, k, v
     if rank == 0 and not args.no_cpu_baseline:
-        rec["cpu_baseline"] = cpu_baseline(cfg, args.cpu_steps, args.scorer)
+        rec["cpu_baseline"], oracle_dec = cpu_baseline(cfg, args.cpu_steps, args.scorer)
+        rec["agreement"] = agreement(gpu_kept, gpu_dec, oracle_dec)
     if rank == 0:
         print(json.dumps(rec), flush=True)
     if world > 1:
@@ -503,7 +648,7 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
     rec = {
         "metric": METRIC, "value": tokens_per_step / (step_ms / 1e3), "unit": "tokens/s",
         "n_gpus": world, "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "scaling": "weak", "vs_baseline": None, "dtype": decode_dtype(cfg),
         "data": "synthetic (seeded counter-based generator)",
         "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
                    "layers": cfg.n_layers, "hidden": cfg.hidden, "kv_heads": cfg.n_kv_heads,
@@ -543,12 +688,17 @@ def run_reference(args):
     rank, _, world = dist_info()
     if rank != 0:
         return
-    from oracle.run import prefill_pair
+    from oracle.run import prefill_pair, prefill_pair_mlstm
     from workload import gen, get_config
     cfg = get_config(args.config)
     if cfg.n_layers != 1:
         raise SystemExit("--impl reference times the oracle on single-layer workloads only")
-    w = gen.scorer_weights(cfg)
+    if args.scorer == "mlstm":
+        mw = gen.mlstm_weights(cfg)
+        prefill = lambda b, h, P: prefill_pair_mlstm(cfg, mw, b, h, P)
+    else:
+        w = gen.scorer_weights(cfg)
+        prefill = lambda b, h, P: prefill_pair(cfg, w, b, h, P)
     L = gen.prompt_lengths(cfg)
     W, K = args.warmup, args.steps
     budget_s = 120.0
@@ -557,7 +707,7 @@ def run_reference(args):
     G = cfg.q_per_kv
     t_setup = time.perf_counter()
     for b, h in pairs:
-        caches.append(prefill_pair(cfg, w, b, h, L[b]))
+        caches.append(prefill(b, h, L[b]))
         q, k, v = gen.decode_inputs(cfg, [L[b]], 0, W + K, b0=b)
         inputs.append((q[:, 0, h * G:(h + 1) * G].double().numpy(), k[:, 0, h].double().numpy(),
                        v[:, 0, h].double().numpy()))
@@ -594,8 +744,7 @@ def run_reference(args):
         "warmup": W, "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded counter-based generator)",
         "impl": "reference",
-        "config": {"workload": f"{cfg.name}: {cfg.description}", "batch": cfg.batch,
-                   "budget_B": cfg.budget_B, "delay_D": cfg.delay_D, "kv_dtype": cfg.kv_dtype},
+        "config": decode_config(cfg, args.scorer, mean_stream_bytes(cfg, L, W, K), world),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                          "sample": (f"each step = one decode step of {n_use} of "
                                     f"{cfg.batch * cfg.n_kv_heads} (sequence, KV head) pairs on one "

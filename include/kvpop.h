@@ -230,8 +230,9 @@ kvpop_status kvpop_prompt_attention(const void* Q_dev, const void* K_dev, const 
                                     float* lse_dev, cudaStream_t stream);
 
 /* First device-side error (a bounded wait that expired) recorded by the
- * cache-free calls kvpop_prompt_attention, kvpop_causal_lse and
- * kvpop_future_target since the last call of this function: KVPOP_OK, or
+ * cache-free calls kvpop_prompt_attention, kvpop_causal_lse,
+ * kvpop_future_target and kvpop_attend_noalloc since the last call of this
+ * function: KVPOP_OK, or
  * KVPOP_ERR_DEVICE_CHECK (details in kvpop_last_error).  Synchronises `stream`
  * and clears the record. */
 kvpop_status kvpop_standalone_status(cudaStream_t stream);
@@ -349,7 +350,12 @@ kvpop_status kvpop_get_pair_state(kvpop_cache* cache, int32_t seq, int32_t head,
  * attributes) with that device current; make that first call before any
  * stream capture.  Every call on a device shares the one array and the array
  * keeps the last call's contents, so calls that overlap on the GPU race:
- * serialise them. */
+ * serialise them.  A bounded wait in the kernel that gives up leaves `out`
+ * incomplete and is reported by the next kvpop_standalone_status (which
+ * synchronises `stream` and allocates nothing); callers that need to know
+ * call it after the attention.  The kernel's shared-memory limit is set to the
+ * device maximum by every path of the library, so caches created on other
+ * threads never lower it under this call. */
 kvpop_status kvpop_attend_noalloc(const void* slotK_dev, const void* slotV_dev,
                                   const void* ringK_dev, const void* ringV_dev,
                                   const int32_t* nvalid_dev, const int32_t* len_dev,

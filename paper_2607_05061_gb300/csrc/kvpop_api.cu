@@ -45,15 +45,21 @@ struct kvpop_cache {
 };
 
 // First device-side error of the cache-free calls (prompt attention, causal LSE,
-// future target); read and cleared by kvpop_standalone_status.
+// future target, allocation-free attention); read and cleared by
+// kvpop_standalone_status.
 __device__ int32_t g_standalone_err[4];
 
-namespace {
-
-int32_t* standalone_err() {
+namespace kvpop {
+// Device address of g_standalone_err on the current device (NULL on failure).
+int32_t* standalone_err_word() {
   void* p = nullptr;
   return cudaGetSymbolAddress(&p, g_standalone_err) == cudaSuccess ? static_cast<int32_t*>(p) : nullptr;
 }
+}  // namespace kvpop
+
+namespace {
+
+int32_t* standalone_err() { return kvpop::standalone_err_word(); }
 
 constexpr uint64_t kMagic = 0x6b7670'6f70'6361ull;   // "kvpopca"
 constexpr uint64_t kStateVersion = 1;
@@ -289,7 +295,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     s = from_cuda(NOTE(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device)));
     const size_t smem = ac.smem_fixed + (pairs + 1) * 4;
     if (s == KVPOP_OK)
-      s = from_cuda(NOTE(cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)));
+      s = from_cuda(NOTE(raise_smem_limit(ac.func, smem)));
     if (s == KVPOP_OK)
       s = from_cuda(NOTE(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, ac.func, ac.threads, smem)));
     if (s == KVPOP_OK && occ < 1) s = KVPOP_ERR_INVALID_ARG;

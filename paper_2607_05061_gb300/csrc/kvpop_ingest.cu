@@ -286,8 +286,8 @@ static size_t ingest_smem(const Dims& dm) {
 cudaError_t prepare_ingest(const Dims& dm) {
   const int smem = (int)ingest_smem(dm);
   if (dm.dtype == KVPOP_F32)
-    return cudaFuncSetAttribute(ingest_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  return cudaFuncSetAttribute(ingest_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return raise_smem_limit(ingest_kernel<float>, smem);
+  return raise_smem_limit(ingest_kernel<bf16>, smem);
 }
 
 cudaError_t launch_ingest(const State& st, const Dims& dm, const void* q, const void* k,

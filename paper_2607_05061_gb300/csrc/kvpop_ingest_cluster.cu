@@ -500,8 +500,8 @@ size_t cluster_ingest_smem(const Dims& dm) {
 cudaError_t prepare_ingest_cluster(const Dims& dm) {
   const int smem = (int)cluster_ingest_smem(dm);
   if (dm.dtype == KVPOP_F32)
-    return cudaFuncSetAttribute(ingest_cluster_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  return cudaFuncSetAttribute(ingest_cluster_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return raise_smem_limit(ingest_cluster_kernel<float>, smem);
+  return raise_smem_limit(ingest_cluster_kernel<bf16>, smem);
 }
 
 template <typename T>

@@ -24,6 +24,21 @@ enum : int {
 // Wall-clock budget of any single mbarrier wait before a kernel gives up.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
+// A kernel's dynamic shared-memory limit is one process-wide attribute.  Every
+// launch path raises it to the device's opt-in maximum -- the same value
+// whoever sets it -- so one caller's set-up never lowers the limit under
+// another caller's launch (caches of different sizes, other host threads).
+// Returns cudaErrorInvalidValue when `need` exceeds that maximum.
+template <typename K>
+inline cudaError_t raise_smem_limit(K* func, size_t need) {
+  int dev = 0, optin = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  if (need > (size_t)optin) return cudaErrorInvalidValue;
+  return cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+}
+
 struct State {                 // device pointers of one cache
   void* slotK;                 // [pairs][B][d]   element type T
   void* slotV;

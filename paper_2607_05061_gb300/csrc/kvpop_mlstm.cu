@@ -463,13 +463,13 @@ cudaError_t prepare_mlstm(const Dims& dm) {
   const int psm = (int)((size_t)2 * dm.d * UTM * 4 + (size_t)UTM * NC * 4);
   cudaError_t e;
   if (dm.dtype == KVPOP_F32) {
-    e = cudaFuncSetAttribute(ingest_mlstm_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, ism);
+    e = raise_smem_limit(ingest_mlstm_kernel<float>, ism);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(mlstm_proj_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, psm);
+      e = raise_smem_limit(mlstm_proj_kernel<float>, psm);
   } else {
-    e = cudaFuncSetAttribute(ingest_mlstm_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, ism);
+    e = raise_smem_limit(ingest_mlstm_kernel<bf16>, ism);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(mlstm_proj_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, psm);
+      e = raise_smem_limit(mlstm_proj_kernel<bf16>, psm);
   }
   return e;
 }

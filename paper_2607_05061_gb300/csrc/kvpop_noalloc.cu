@@ -14,12 +14,18 @@
 // All calls on a device share it and it keeps the last call's contents, so
 // calls that overlap on the GPU (different streams, or different threads
 // without ordering) race on it; callers must serialise them.
+//
+// A bounded wait inside the kernel that gives up is recorded in the library's
+// device error word of the cache-free calls, which kvpop_standalone_status reads
+// and clears (that word is a __device__ variable too: reading it allocates
+// nothing).
 #include <mutex>
 
 #include "kvpop_internal.cuh"
 
 namespace kvpop {
 void note_error(const char* msg);
+int32_t* standalone_err_word();
 }
 
 using namespace kvpop;
@@ -35,14 +41,16 @@ constexpr int kMaxPairs = 12288;
 struct DeviceSetup {
   bool ready = false;
   unsigned char* scratch = nullptr;   // device address of g_attend_scratch
+  int32_t* err = nullptr;             // device address of the cache-free calls' error word
   int sms = 0;
   int smem_optin = 0;
 };
 DeviceSetup g_setup[kMaxDevices];
 std::mutex g_setup_mu;
 
-// First use on a device, with that device current: resolve the array's device
-// address and allow the attention kernels their dynamic shared memory.
+// First use on a device, with that device current: resolve the device
+// addresses of the array and of the error word, and allow the attention
+// kernels their dynamic shared memory.
 kvpop_status setup_device(int dev, DeviceSetup** out) {
   std::lock_guard<std::mutex> lock(g_setup_mu);
   DeviceSetup& s = g_setup[dev];
@@ -51,6 +59,11 @@ kvpop_status setup_device(int dev, DeviceSetup** out) {
     cudaError_t e = cudaGetSymbolAddress(&ptr, g_attend_scratch);
     if (e != cudaSuccess) {
       note_error("kvpop_attend_noalloc: cudaGetSymbolAddress of the scratch array failed");
+      return KVPOP_ERR_CUDA;
+    }
+    int32_t* err = standalone_err_word();
+    if (!err) {
+      note_error("kvpop_attend_noalloc: cudaGetSymbolAddress of the error word failed");
       return KVPOP_ERR_CUDA;
     }
     int sms = 0, optin = 0;
@@ -65,14 +78,14 @@ kvpop_status setup_device(int dev, DeviceSetup** out) {
           dm.G = G;
           AttendConfig ac;
           if (e == cudaSuccess) e = attend_config(dm, &ac);
-          if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+          if (e == cudaSuccess) e = raise_smem_limit(ac.func, 0);
         }
     if (e != cudaSuccess) {
       note_error("kvpop_attend_noalloc: device set-up failed");
       return KVPOP_ERR_CUDA;
     }
     s.scratch = static_cast<unsigned char*>(ptr);
+    s.err = err;
     s.sms = sms;
     s.smem_optin = optin;
     s.ready = true;
@@ -125,8 +138,7 @@ extern "C" kvpop_status kvpop_attend_noalloc(const void* slotK, const void* slot
   const int grid = ds->sms;                       // one CTA per SM (the kernel's launch bounds)
   const size_t count_bytes = ((size_t)pairs * 4 + 255) & ~size_t(255);
   const size_t part_bytes = (size_t)2 * grid * (q_per_kv * head_dim + 2 * q_per_kv) * 4;
-  const size_t err_bytes = 256;
-  if (count_bytes + part_bytes + err_bytes > kScratchBytes) {
+  if (count_bytes + part_bytes > kScratchBytes) {
     note_error("kvpop_attend_noalloc: split-K scratch would exceed the fixed 2 MiB array");
     return KVPOP_ERR_INVALID_ARG;
   }
@@ -140,13 +152,9 @@ extern "C" kvpop_status kvpop_attend_noalloc(const void* slotK, const void* slot
   s.len = const_cast<int32_t*>(len);
   s.part_count = reinterpret_cast<int32_t*>(ds->scratch);
   s.part = reinterpret_cast<float*>(ds->scratch + count_bytes);
-  s.err = reinterpret_cast<int32_t*>(ds->scratch + count_bytes + part_bytes);
-  // another cache in this process may have lowered the kernel's shared-memory limit
-  cudaError_t e = cudaFuncSetAttribute(ac.func, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       ds->smem_optin);
+  s.err = ds->err;     // first error wins; kvpop_standalone_status reads and clears it
   // the counters must start at zero; the array keeps whatever the last call left
-  if (e == cudaSuccess) e = cudaMemsetAsync(s.part_count, 0, count_bytes, stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(s.err, 0, 64, stream);
+  cudaError_t e = cudaMemsetAsync(s.part_count, 0, count_bytes, stream);
   if (e == cudaSuccess) e = launch_attend(s, dm, q, out, grid, stream);
   if (e != cudaSuccess) {
     note_error("kvpop_attend_noalloc: launch failed");

@@ -553,16 +553,16 @@ cudaError_t prepare_prefill(const Dims& dm) {
   const int smem = (int)score_smem(dm);
   cudaError_t e;
   if (dm.dtype == KVPOP_F32)
-    e = cudaFuncSetAttribute(prefill_score_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = raise_smem_limit(prefill_score_kernel<float>, smem);
   else
-    e = cudaFuncSetAttribute(prefill_score_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = raise_smem_limit(prefill_score_kernel<bf16>, smem);
   if (e != cudaSuccess || !gemm_ok(dm)) return e;
   const int gs = (int)gemm_smem(dm);
   if (dm.dtype == KVPOP_F32)
-    return dm.F == 256 ? cudaFuncSetAttribute(prefill_score_gemm_kernel<float, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs)
-                       : cudaFuncSetAttribute(prefill_score_gemm_kernel<float, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs);
-  return dm.F == 256 ? cudaFuncSetAttribute(prefill_score_gemm_kernel<bf16, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs)
-                     : cudaFuncSetAttribute(prefill_score_gemm_kernel<bf16, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, gs);
+    return dm.F == 256 ? raise_smem_limit(prefill_score_gemm_kernel<float, 16>, gs)
+                       : raise_smem_limit(prefill_score_gemm_kernel<float, 8>, gs);
+  return dm.F == 256 ? raise_smem_limit(prefill_score_gemm_kernel<bf16, 16>, gs)
+                     : raise_smem_limit(prefill_score_gemm_kernel<bf16, 8>, gs);
 }
 
 template <typename T>

@@ -374,7 +374,7 @@ template <typename Kern>
 cudaError_t launch_cfg(Kern k, dim3 grid, int threads, size_t smem, cudaStream_t stream,
                        const PromptArgs& a) {
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit(k, smem);
     if (e != cudaSuccess) return e;
   }
   k<<<grid, threads, smem, stream>>>(a);

@@ -346,7 +346,7 @@ template <int G, bool DENSE, bool WANT_Y, int ST>
 cudaError_t launch_t5_st(const PromptArgs& a, int n_pairs, size_t smem, cudaStream_t stream) {
   constexpr int BM = T5_ROWS / G;
   auto k = prompt_t5_kernel<G, DENSE, WANT_Y, ST>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = raise_smem_limit(k, smem);
   if (e != cudaSuccess) return e;
   dim3 grid((a.S + BM - 1) / BM, n_pairs);
   k<<<grid, T5_THREADS, smem, stream>>>(a);

@@ -361,7 +361,7 @@ template <typename T, int F, int G>
 cudaError_t launch_g(const CUtensorMap* maps, const ScArgs& a, int n_pairs, cudaStream_t stream) {
   const ScOff off = sc_offsets(F, a.D);
   auto k = score_tf32_kernel<T, F, G>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, off.total);
+  cudaError_t e = raise_smem_limit(k, off.total);
   if (e != cudaSuccess) return e;
   dim3 grid((a.Pmax + SC_M - 1) / SC_M, n_pairs);
   k<<<grid, SC_THREADS, off.total, stream>>>(maps[0], maps[1], a);

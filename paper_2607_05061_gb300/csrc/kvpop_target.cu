@@ -581,13 +581,13 @@ cudaError_t launch_future_target(const void* Q, const void* K, const float* lse,
     dim3 grid((S + T6_ROWS - 1) / T6_ROWS, n_pairs);
     cudaError_t e = cudaSuccess;
     if (G == 4) {
-      e = cudaFuncSetAttribute(target_t5_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      e = raise_smem_limit(target_t5_kernel<4>, T6_SMEM);
       if (e == cudaSuccess) target_t5_kernel<4><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
     } else if (G == 2) {
-      e = cudaFuncSetAttribute(target_t5_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      e = raise_smem_limit(target_t5_kernel<2>, T6_SMEM);
       if (e == cudaSuccess) target_t5_kernel<2><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
     } else {
-      e = cudaFuncSetAttribute(target_t5_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, T6_SMEM);
+      e = raise_smem_limit(target_t5_kernel<1>, T6_SMEM);
       if (e == cudaSuccess) target_t5_kernel<1><<<grid, T6_THREADS, T6_SMEM, stream>>>(a);
     }
     if (e != cudaSuccess) return e;
@@ -595,13 +595,11 @@ cudaError_t launch_future_target(const void* Q, const void* K, const float* lse,
     const size_t smem = d == 128 ? TgP<128>::SMEM : TgP<64>::SMEM;
     dim3 grid((S + TgP<128>::ROWS - 1) / TgP<128>::ROWS, n_pairs);
     if (d == 128) {
-      cudaError_t e = cudaFuncSetAttribute(target_tc_kernel<128>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaError_t e = raise_smem_limit(target_tc_kernel<128>, smem);
       if (e != cudaSuccess) return e;
       target_tc_kernel<128><<<grid, TgP<128>::THREADS, smem, stream>>>(a);
     } else {
-      cudaError_t e = cudaFuncSetAttribute(target_tc_kernel<64>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaError_t e = raise_smem_limit(target_tc_kernel<64>, smem);
       if (e != cudaSuccess) return e;
       target_tc_kernel<64><<<grid, TgP<64>::THREADS, smem, stream>>>(a);
     }

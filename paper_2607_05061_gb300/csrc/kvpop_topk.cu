@@ -319,7 +319,7 @@ cudaError_t launch_topk(const float* prio, const int32_t* len, int rows_per_len,
   const int split = std::max(1, std::min(want, S / (nch * 512)));
   const int chunk = (S + nch * split - 1) / (nch * split);
   const size_t smem = (size_t)nch * words_bytes;
-  e = cudaFuncSetAttribute(cutoff_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  e = raise_smem_limit(cutoff_kernel, smem);
   if (e != cudaSuccess) return e;
   CutArgs ca{rank, len, rows_per_len, n_rows, S, s, w, k, tau};
   cutoff_kernel<<<dim3(n_rows, split), nch * 32, smem, stream>>>(ca, chunk);

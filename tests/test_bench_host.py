@@ -118,6 +118,12 @@ def test_reference_arm_prints_one_contract_line(workload):
     # the same metric as the GPU arm of that workload
     want = bench.METRIC if workload == "decode" else bench.prompt_metric(workload)[0]
     assert recs[0]["metric"] == want
+    if workload == "decode":
+        # and the same config object the GPU arm prints for these steps
+        from workload import gen
+        cfg = get_config("tiny")
+        L = gen.prompt_lengths(cfg)
+        assert recs[0]["config"] == bench.decode_config(cfg, "mlp", bench.mean_stream_bytes(cfg, L, 3, 2), 1)
 
 
 def test_reference_arm_under_torchrun_prints_once_from_rank0():
@@ -157,3 +163,39 @@ def test_target_flops_count_key_query_pairs(P, D):
     pairs = sum(1 for t in range(P) for d in range(P) if d >= t + D)
     want = 2.0 * cfg.head_dim * cfg.q_per_kv * cfg.n_kv_heads * pairs
     assert bench.target_flops(cfg, [P]) == want
+
+
+# ---------------------------------------------------------------- decode line: L2 rule, dtype, agreement
+def test_l2_flush_only_for_workloads_smaller_than_twice_l2():
+    from workload import gen
+    for name, want in (("q4b", True), ("cr8x", False), ("ragged", False), ("tiny", True)):
+        cfg = get_config(name)
+        L = gen.prompt_lengths(cfg)
+        assert bench.flushes_l2(bench.kv_stream_bytes(cfg, L, 0)) is want, name
+    assert bench.decode_dtype(get_config("cr8x")) == "bf16 (fp32 accumulate)"
+    assert bench.decode_dtype(get_config("tiny")) == "f32"
+
+
+def test_agreement_counts_decisions_and_kept_sets():
+    gpu_dec = [[[(0, -1), (3, 7)]], [[(-1, -1), (2, 9)]]]          # [step][b][h]
+    oracle = {(0, 0): ([1, 2], [(0, -1), (-1, -1)]),
+              (0, 1): ([4, 5], [(3, 7), (2, 8)])}
+    gpu_kept = {(0, 0): [2, 1], (0, 1): [4, 6]}
+    a = bench.agreement(gpu_kept, gpu_dec, oracle)
+    assert a["decisions"] == 4 and a["decode_decisions_equal"] == 0.75
+    assert a["prefill_kept_sets_equal"] == 0.5 and a["pairs"] == 2 and a["steps"] == 2
+    assert a["first_mismatch"] == {"pair": [0, 1], "step": 1, "gpu": [2, 9], "oracle": [2, 8]}
+
+
+def test_oracle_pair_job_reports_the_oracle_decisions():
+    from oracle.run import run_pair
+    from workload import gen
+    cfg = get_config("tiny")
+    L = gen.prompt_lengths(cfg)
+    t, kept, dec = bench._oracle_pair_job(("tiny", 0, 1, 12, "mlp"))
+    tr = run_pair(cfg, gen.scorer_weights(cfg), 0, 1, L[0], 12, attend=False, keep_cache=True)
+    assert t > 0
+    assert dec == list(zip(tr.slots, tr.evicted))
+    assert any(e >= 0 for _, e in dec)
+    ref = run_pair(cfg, gen.scorer_weights(cfg), 0, 1, L[0], 0, keep_cache=True)
+    assert kept == ref.cache.kept_positions()

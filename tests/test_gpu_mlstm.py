@@ -91,3 +91,41 @@ def test_mlstm_checkpoint_resume_is_bit_identical(cuda_device):
     assert np.array_equal(ga.outputs, gb.outputs)
     a.free()
     b.free()
+
+
+def test_mlstm_full_size_sampled(cuda_device):
+    """cr8x shape (P 32768, B 4096, D 16) with the mLSTM scorer, on sampled pairs the
+    oracle computes in full: bit-exact evictions and attention with injected scores,
+    then the GPU recurrence's own scores against the oracle's."""
+    cfg = get_config("cr8x", batch=8)
+    mw = gen.mlstm_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    steps = 24
+    sample = [(0, 0), (5, 3), (7, 7)]
+    pov = injected_prefill_scores(cfg, max(L), "cpu")
+    dov = injected_decode_scores(cfg, steps, "cpu")
+    cache = make_cache(cfg, None, mlstm=mw)
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device), sample=sample)
+    ref = oracle_pairs(cfg, None, L, steps, sample, prefill_override=pov, decode_override=dov,
+                       mlstm=mw)
+    err = compare(cfg, g, ref, sample)
+    print(f"mlstm cr8x injected: max-abs attention error {err:.3e}")
+    assert err <= TOL[cfg.kv_dtype]
+    cache.free()
+    # own scores: the recurrence over the whole 32768-token prompt, then decode
+    cache = make_cache(cfg, None, mlstm=mw)
+    gpu_prefill(cache, cfg, L, cuda_device)
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, sample=sample)
+    ref = oracle_pairs(cfg, None, L, steps, sample, mlstm=mw, attend=False)
+    worst = 0.0
+    for (b, h), tr in zip(sample, ref):
+        want = np.asarray(tr.scores, dtype=np.float64)
+        got = g.scores[:, b, h].astype(np.float64)
+        worst = max(worst, float(np.max(np.abs(got - want) / (1.0 + np.abs(want)))))
+        ev = g.evict[:, b, h]
+        same = (ev[:, 0] == np.asarray(tr.slots)) & (ev[:, 1] == np.asarray(tr.evicted))
+        print(f"mlstm cr8x {(b, h)}: decode eviction agreement {same.mean():.4f}")
+    print(f"mlstm cr8x: worst relative decode score error {worst:.2e}")
+    assert worst <= 1e-4
+    cache.free()

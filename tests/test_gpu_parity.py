@@ -185,7 +185,10 @@ def test_full_size_gpu_scorer(cuda_device):
     for (b, h), tr in zip(sample, ref):
         want = np.asarray(tr.scores, dtype=np.float64)
         got = g.scores[:, b, h].astype(np.float64)
-        assert np.all(np.abs(got - want) <= 5e-5 * (1.0 + np.abs(want)))
+        # the same fp32-accurate bound as the other scorer checks (3xTF32 hidden slice)
+        rel = np.abs(got - want) / (1.0 + np.abs(want))
+        print(f"cr8x GPU scorer {(b, h)}: max relative score error {np.nanmax(rel):.2e}")
+        assert np.all(rel <= 2e-5)
         pos, sc = cache.pair_state(b, h)
         o = set(tr.cache.kept_positions())
         # end-to-end decisions with each side's own scores: reported, not gated

@@ -5,8 +5,9 @@ tolerance on sampled pairs (first, last and one in between), after a prompt that
 already overflows the budget.  One pair more is rejected by kvpop_init_cache (a
 host-side check, tests/test_abi_host.py).
 
-This file is named to be collected last, so a run that stops at the first failure
-has run every other test before it."""
+This file is named to be collected after the other parity tests (only the
+allocation-free attention's test comes later), so a run that stops at the first
+failure has run them before this large case."""
 import pytest
 
 from gpu_harness import (TOL, compare, gpu_decode, gpu_prefill, injected_decode_scores,
