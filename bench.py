@@ -31,7 +31,6 @@ import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
-ATTN_SAMPLE = 16          # decode steps per attention-duration sample
 sys.path.insert(0, ROOT)
 
 METRIC = "decode tokens/sec at 1 GB300 (batch x steps) and achieved HBM GB/s"
@@ -106,7 +105,7 @@ def kv_stream_bytes(cfg, lengths, step: int) -> int:
 
 L2_BYTES = 129e6           # GB300 L2 (126 MiB)
 FLUSH_BYTES = 512 << 20    # written between timed steps whose inputs fit in twice the L2
-ATTN_POST_LAUNCHES = 32    # event-timed attention launches after a short timed region
+ATTN_POST_LAUNCHES = 32    # event-timed attention launches after the timed region
 
 
 def flushes_l2(bytes_per_step: float) -> bool:
@@ -380,8 +379,8 @@ def run_kvpop(args):
     bytes_per_launch = mean_stream_bytes(cfg, L, W, K)
     flush = flushes_l2(bytes_per_launch)
     flush_buf = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev) if flush else None
-    post = ATTN_POST_LAUNCHES if (K < 64 or flush) else 0
-    q, k, v = gen.decode_inputs(cfg, L, 0, W + K + post, device=dev)
+    post = ATTN_POST_LAUNCHES
+    q, k, v = gen.decode_inputs(cfg, L, 0, W + K + post + 2, device=dev)
     out = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     for j in range(W):
@@ -392,36 +391,46 @@ def run_kvpop(args):
     def ev():
         return torch.cuda.Event(enable_timing=True)
 
-    # The attention kernel's own duration: with a long timed region, events around it on
-    # every ATTN_SAMPLE-th step (events between the ingest and the attention stop the
-    # attention from launching as a programmatic dependent of the ingest, so the other
-    # steps run without them); with a short one, or with L2 flushes, in a loop of
-    # ATTN_POST_LAUNCHES steps after it with events around each attention.
-    samples = [] if post else list(range(0, K, ATTN_SAMPLE))
-    ev_s = {i: ev() for i in samples}
-    ev_e = {i: ev() for i in samples}
+    def capture(body):
+        """One CUDA graph of the library calls `body` makes (nothing runs while capturing)."""
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(g, stream=side):
+                body()
+        stream.wait_stream(side)
+        return g
+
+    # Inputs larger than L2: the K timed steps are replayed from one CUDA graph between
+    # two events on the stream, so the device runs them back to back (in an eager loop
+    # the first steps also wait for the host to enqueue them).  Inputs smaller than twice
+    # L2: an eager loop writes the flush buffer before every step and brackets each step
+    # with its own events; the flush gives the host time to enqueue the step.
     step_ev = [(ev(), ev()) for _ in range(K)] if flush else []
     t_start, t_end = ev(), ev()
+    graph = None
+    if not flush:
+        def timed_body():
+            for i in range(K):
+                cache.ingest(q[W + i], k[W + i], v[W + i])
+                cache.attend(q[W + i], out)
+        graph = capture(timed_body)
     clocks = ClockSampler(local_rank)
     clocks.start()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     t_start.record(stream)
-    for i in range(K):
-        j = W + i
-        if flush:
+    if flush:
+        for i in range(K):
             flush_buf.fill_(float(i))
             step_ev[i][0].record(stream)
-        cache.ingest(q[j], k[j], v[j])
-        if i in ev_s:
-            ev_s[i].record(stream)
-            cache.attend(q[j], out)
-            ev_e[i].record(stream)
-        else:
-            cache.attend(q[j], out)
-        if flush:
+            cache.ingest(q[W + i], k[W + i], v[W + i])
+            cache.attend(q[W + i], out)
             step_ev[i][1].record(stream)
+    else:
+        graph.replay()
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -432,33 +441,34 @@ def run_kvpop(args):
         step_ms_local = statistics.mean(a.elapsed_time(b) for a, b in step_ev)
     else:
         step_ms_local = t_start.elapsed_time(t_end) / K
-    attn_pairs = []
-    if post:
-        for i in range(post):
-            j = W + K + i
-            cache.ingest(q[j], k[j], v[j])
-            if flush:
-                flush_buf.fill_(float(i))
-            a, b = ev(), ev()
-            a.record(stream)
-            cache.attend(q[j], out)
-            b.record(stream)
-            attn_pairs.append((a, b))
-        torch.cuda.synchronize()
-        attn_ms = statistics.mean(a.elapsed_time(b) for a, b in attn_pairs)
-        attn_bytes = mean_stream_bytes(cfg, L, W + K, post)
-        attn_how = (f"CUDA events around the attention in {post} decode steps after the timed "
-                    f"region (the ingest between them untimed" +
-                    (", L2 flushed before each)" if flush else ")"))
-    else:
-        attn_ms = statistics.mean(ev_s[i].elapsed_time(ev_e[i]) for i in samples)
-        attn_bytes = statistics.mean(kv_stream_bytes(cfg, L, W + i) for i in samples)
-        attn_how = (f"CUDA events around the attention on {len(samples)} of the {K} timed steps "
-                    f"(every {ATTN_SAMPLE}th)")
+    del graph
+    # The attention kernel's own duration: ATTN_POST_LAUNCHES further decode steps with
+    # events around each attention (events between the ingest and the attention stop the
+    # attention from launching as a programmatic dependent of the ingest, which is why
+    # the timed steps carry none); the first two, which wait for the host to enqueue
+    # them after the synchronisation, are not counted.
+    attn_ev = []
+    for i in range(post + 2):
+        j = W + K + i
+        cache.ingest(q[j], k[j], v[j])
+        if flush:
+            flush_buf.fill_(float(i))
+        a, b = ev(), ev()
+        a.record(stream)
+        cache.attend(q[j], out)
+        b.record(stream)
+        attn_ev.append((a, b))
+    torch.cuda.synchronize()
+    cache.check()
+    attn_ms = statistics.mean(a.elapsed_time(b) for a, b in attn_ev[2:])
+    attn_bytes = mean_stream_bytes(cfg, L, W + K + 2, post)
+    attn_how = (f"CUDA events around the attention in {post} decode steps after the timed "
+                f"region (the ingest between them untimed" +
+                (", L2 flushed before each)" if flush else ")"))
 
     # end to end through the C ABI on host buffers (pinned), copies inside the timed region
     E = max(1, args.e2e_steps)
-    s0 = W + K + post
+    s0 = W + K + post + 2
     qa, ka, va = gen.decode_inputs(cfg, L, s0, E, device="cpu")
     # each step's q, k, v back to back in one pinned buffer (one host-to-device copy)
     qb, kb = qa[0].numel() * qa.element_size(), ka[0].numel() * ka.element_size()

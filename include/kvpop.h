@@ -124,7 +124,8 @@ kvpop_status kvpop_init_cache(const kvpop_config* cfg, const kvpop_scorer* score
 /* As kvpop_init_cache with the mLSTM scorer; cfg->scorer_hidden is ignored.
  * The cache additionally holds the recurrent state (C, z, m) of every
  * (sequence, KV head), which prefill builds over the prompt and every decode
- * step advances by one token (a sequential scan per pair in prefill). */
+ * step advances by one token (in prefill, the chunkwise form of the recurrence:
+ * 64-token chunks one after another per pair, the tokens of a chunk together). */
 kvpop_status kvpop_init_cache_mlstm(const kvpop_config* cfg, const kvpop_mlstm_scorer* scorer,
                                     cudaStream_t stream, kvpop_cache** out);
 
@@ -371,6 +372,16 @@ const char* kvpop_last_error(void);
 /* Testing hook: make the n-th device allocation from now fail (n >= 1), or
  * disable with n <= 0.  Affects only this library's allocations. */
 void kvpop_debug_fail_alloc_after(int32_t n);
+
+/* Testing hook for the failure path of the bounded device waits (no counterpart in
+ * the paper): while `on` is non-zero, the copy-issuing thread of the bf16
+ * tensor-core decode attention (kvpop_decode_attend, kvpop_decode_step) neither
+ * arms a barrier nor issues a copy, so every consumer's first wait runs out after
+ * the kernels' wait limit (2 s), records a timeout and skips the rest of its work;
+ * `out` is then unspecified and the next kvpop_check returns
+ * KVPOP_ERR_DEVICE_CHECK.  Nothing faults and no copy is in flight when the kernel
+ * ends.  Affects launches made after the call; 0 (the default) turns it off. */
+void kvpop_debug_skip_attention_copies(int32_t on);
 
 #ifdef __cplusplus
 }

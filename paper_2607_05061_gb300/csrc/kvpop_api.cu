@@ -50,6 +50,7 @@ struct kvpop_cache {
 __device__ int32_t g_standalone_err[4];
 
 namespace kvpop {
+extern int g_debug_skip_copies;   // kvpop_attend_tc.cu
 // Device address of g_standalone_err on the current device (NULL on failure).
 int32_t* standalone_err_word() {
   void* p = nullptr;
@@ -222,6 +223,8 @@ const char* kvpop_status_string(kvpop_status s) {
 }
 
 void kvpop_debug_fail_alloc_after(int32_t n) { g_fail_after = n > 0 ? n : 0; }
+
+void kvpop_debug_skip_attention_copies(int32_t on) { kvpop::g_debug_skip_copies = on ? 1 : 0; }
 
 const char* kvpop_last_error(void) { return g_last_error; }
 

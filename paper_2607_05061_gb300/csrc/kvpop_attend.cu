@@ -184,7 +184,8 @@ __global__ void __launch_bounds__(Traits<T, HD, G>::THREADS, 1) attend_kernel(At
     const int per = (npairs + NT - 1) / NT;
     const int beg = min(tid * per, npairs), end = min(beg + per, npairs);
     int local = 0;
-    for (int i = beg; i < end; ++i) local += tiles_of(a.nvalid[i], min(a.len[i], a.D), TILE);
+    for (int i = beg; i < end; ++i)
+      local += tiles_of(used_slots(a.nvalid[i], a.B, a.err), window_rows(a.len[i], a.D, a.err), TILE);
     int incl = local;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -211,7 +212,7 @@ __global__ void __launch_bounds__(Traits<T, HD, G>::THREADS, 1) attend_kernel(At
     int run = scan[warp] + incl - local;
     for (int i = beg; i < end; ++i) {
       prefix[i] = run;
-      run += tiles_of(a.nvalid[i], min(a.len[i], a.D), TILE);
+      run += tiles_of(used_slots(a.nvalid[i], a.B, nullptr), window_rows(a.len[i], a.D, nullptr), TILE);
     }
     __syncthreads();
   }
@@ -243,7 +244,7 @@ __global__ void __launch_bounds__(Traits<T, HD, G>::THREADS, 1) attend_kernel(At
       for (long long t = t0; t < t1; ++t, ++i) {
         while (t >= prefix[p + 1]) ++p;
         const int lt = (int)(t - prefix[p]);
-        const int nv = a.nvalid[p];
+        const int nv = used_slots(a.nvalid[p], a.B, nullptr);
         const int nvt = (nv + TILE - 1) / TILE;
         const unsigned char *sk, *sv;
         int cnt;
@@ -254,7 +255,7 @@ __global__ void __launch_bounds__(Traits<T, HD, G>::THREADS, 1) attend_kernel(At
           sv = a.slotV + ((size_t)p * a.B + k0) * R;
         } else {
           const int k0 = (lt - nvt) * TILE;
-          cnt = min(TILE, min(a.len[p], a.D) - k0);
+          cnt = min(TILE, window_rows(a.len[p], a.D, nullptr) - k0);
           sk = a.ringK + ((size_t)p * a.D + k0) * R;
           sv = a.ringV + ((size_t)p * a.D + k0) * R;
         }

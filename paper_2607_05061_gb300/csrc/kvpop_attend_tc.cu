@@ -74,6 +74,7 @@ struct TcArgs {
   int pairs, B, D;
   int ring_rows;               // rows of a window box: min(TILE, D rounded up to 8)
   float qscale;
+  int skip_copies;             // testing hook: the producer issues nothing (see below)
 };
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
@@ -154,7 +155,7 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
   // Launched as a programmatic dependent of the ingest: everything below reads the
   // state it writes, so wait here for it to complete (a no-op without a predecessor).
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  build_schedule<NT>(a.nvalid, a.len, npairs, a.D, TILE, prefix, scan);
+  build_schedule<NT>(a.nvalid, a.len, npairs, a.B, a.D, TILE, prefix, scan, a.err);
   const long long Ttot = prefix[npairs];
   if (Ttot <= 0) return;
   const long long NC = min((long long)gridDim.x, Ttot);
@@ -175,14 +176,17 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
   }
 
   // ---- producer -------------------------------------------------------------------
+  // With the testing hook on, the producer neither arms a barrier nor issues a copy:
+  // every consumer's first bounded wait runs out, records DEVERR_TIMEOUT_FULL and the
+  // consumers skip the rest of their work; no copy is in flight when the CTA exits.
   if (warp == NWC) {
-    if (lane == 0) {
+    if (lane == 0 && !a.skip_copies) {
       int p = p0;
       long long i = 0;
       for (long long t = t0; t < t1; ++t, ++i) {
         while (t >= prefix[p + 1]) ++p;
         const int lt = (int)(t - prefix[p]);
-        const int nv = a.nvalid[p];
+        const int nv = used_slots(a.nvalid[p], a.B, nullptr);
         const int nvt = (nv + TILE - 1) / TILE;
         const CUtensorMap *mk, *mv;
         int row;
@@ -287,10 +291,11 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     const int s = (int)(i % STAGES);
     if (ok) ok = mbar_wait(smem_u32(&bars[s]), (uint32_t)((i / STAGES) & 1), a.err, DEVERR_TIMEOUT_FULL);
     const int lt = (int)(t - prefix[p]);
-    const int nv = a.nvalid[p];
+    const int nv = used_slots(a.nvalid[p], a.B, nullptr);
     const int nvt = (nv + TILE - 1) / TILE;
     const int cnt = lt < nvt ? min(TILE, nv - lt * TILE)
-                             : min(TILE, min(a.len[p], a.D) - (lt - nvt) * TILE);
+                             : min(TILE, window_rows(a.len[p], a.D, nullptr) - (lt - nvt) * TILE);
+    dcheck(cnt > 0 && cnt <= TILE, a.err, DEVERR_INDEX);
     const int key0 = warp * 16;
     if (ok && key0 < cnt) {
       const uint32_t kbase = smem_u32(smem + (size_t)s * Tr::STAGE_BYTES);
@@ -400,6 +405,8 @@ struct TcMaps {
   CUtensorMap sk, sv, rk, rv;
 };
 
+int g_debug_skip_copies = 0;   // kvpop_debug_skip_attention_copies
+
 // Window boxes only need D rows (rounded up to a swizzle atom's 8) when D < TILE.
 static int tc_ring_rows(const Dims& dm) {
   const int tile = TcTraits<128, 4>::TILE;
@@ -459,6 +466,7 @@ cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const v
   a.D = dm.D;
   a.ring_rows = tc_ring_rows(dm);
   a.qscale = kLog2e / sqrtf((float)dm.d);
+  a.skip_copies = g_debug_skip_copies;
   // programmatic stream serialisation: the grid may be scheduled while the kernel
   // before it (the ingest) finishes; the kernel waits for it before touching the state
   cudaLaunchConfig_t cfg = {};

@@ -32,8 +32,10 @@ __device__ __forceinline__ void evict_and_scatter(const State& st, const Dims& d
     slot = nv;
   } else if (prio > st.min_score[pair]) {
     slot = st.min_slot[pair];
-    evicted = ps[slot];
+    if (!dcheck(slot >= dm.s && slot < B, st.err, DEVERR_INDEX)) slot = -1;
+    else evicted = ps[slot];
   }
+  if (slot >= 0 && !dcheck(nv >= 0, st.err, DEVERR_INDEX)) slot = -1;
   if (slot >= 0) {
     T* dk = static_cast<T*>(st.slotK) + ((size_t)pair * B + slot) * d;
     T* dv = static_cast<T*>(st.slotV) + ((size_t)pair * B + slot) * d;

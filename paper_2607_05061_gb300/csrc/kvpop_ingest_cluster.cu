@@ -425,6 +425,9 @@ __global__ void __launch_bounds__(NT, 1) ingest_cluster_kernel(ClArgs<T> a) {
     slot = ev_mslot;
     evicted = reg_min ? ev_pos : ps[slot];
   }
+  if (slot >= 0 && !dcheck(slot < B && ev_nv >= 0 && (ev_nv < B || slot >= dm.s), a.st.err,
+                           DEVERR_INDEX))
+    slot = -1;
   if (slot >= 0) {
     T* dk = static_cast<T*>(a.st.slotK) + ((size_t)pair * B + slot) * d;
     T* dv = static_cast<T*>(a.st.slotV) + ((size_t)pair * B + slot) * d;

@@ -19,24 +19,56 @@ enum : int {
   DEVERR_TIMEOUT_EMPTY = 2,    // producer gave up waiting for a free stage
   DEVERR_TIMEOUT_DRAIN = 3,    // producer gave up draining its copies at exit
   DEVERR_BAD_SCHEDULE = 4,     // attention schedule inconsistent with the state
+  DEVERR_INDEX = 5,            // an index check failed (device-check build only)
 };
+
+// Index checks of the device-check build (compiled with -DKVPOP_DEVICE_CHECKS):
+// dcheck(cond, err, code) records `code` in *err (first error wins) and returns
+// false when cond fails, so the caller skips the access instead of trapping.  In
+// the normal build it is `true` and compiles away.
+#ifdef KVPOP_DEVICE_CHECKS
+__device__ __forceinline__ bool dcheck(bool cond, int32_t* err, int code) {
+  if (!cond && err) atomicCAS(err, 0, code);
+  return cond;
+}
+#else
+__device__ __forceinline__ bool dcheck(bool, int32_t*, int) { return true; }
+#endif
+
+// Used slots and window rows of a pair, clamped to the buffers they index, so that
+// state the library did not write (the allocation-free entry point takes it from the
+// caller) can never send a copy outside them; the device-check build also records
+// any value that needed clamping.
+__device__ __forceinline__ int used_slots(int nv, int B, int32_t* err) {
+  dcheck(nv >= 0 && nv <= B, err, DEVERR_INDEX);
+  return min(max(nv, 0), B);
+}
+__device__ __forceinline__ int window_rows(int len, int D, int32_t* err) {
+  dcheck(len >= 0, err, DEVERR_INDEX);
+  return min(max(len, 0), D);
+}
+
 
 // Wall-clock budget of any single mbarrier wait before a kernel gives up.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
 // A kernel's dynamic shared-memory limit is one process-wide attribute.  Every
-// launch path raises it to the device's opt-in maximum -- the same value
-// whoever sets it -- so one caller's set-up never lowers the limit under
-// another caller's launch (caches of different sizes, other host threads).
-// Returns cudaErrorInvalidValue when `need` exceeds that maximum.
+// launch path raises it to the most the device allows that kernel (the opt-in
+// maximum less its static shared memory) -- the same value whoever sets it --
+// so one caller's set-up never lowers the limit under another caller's launch
+// (caches of different sizes, other host threads).  Returns
+// cudaErrorInvalidValue when `need` exceeds that maximum.
 template <typename K>
 inline cudaError_t raise_smem_limit(K* func, size_t need) {
   int dev = 0, optin = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  cudaFuncAttributes fa;
+  if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, reinterpret_cast<const void*>(func));
   if (e != cudaSuccess) return e;
-  if (need > (size_t)optin) return cudaErrorInvalidValue;
-  return cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+  const long long room = (long long)optin - (long long)fa.sharedSizeBytes;
+  if (room < 0 || (long long)need > room) return cudaErrorInvalidValue;
+  return cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)room);
 }
 
 struct State {                 // device pointers of one cache

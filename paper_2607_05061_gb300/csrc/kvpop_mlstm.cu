@@ -355,94 +355,285 @@ struct MScanArgs {
   int first_seq, Pmax, NF;
 };
 
-// One CTA per (sequence, head): the recurrence over the prompt, scoring every
-// u = t - D right after token t has been absorbed.
-__global__ void __launch_bounds__(NTM) mlstm_scan_kernel(MScanArgs a) {
+// Chunkwise form of the same recurrence (App. A: the mLSTM as linear attention with
+// gates).  Within a chunk of L tokens starting at t0, with F_s the cumulative log
+// forget gate of the chunk up to token s and g_s = log i_s - F_s, the state after
+// absorbing token t is, up to one common scale,
+//   C(t) = e^{m - R_t} C + sum_{s <= t} e^{g_s - R_t} k~_s v~_s^T,   R_t = max(m, max_{s<=t} g_s)
+// (same for z), where (C, z, m) is the stabilised state at the chunk start; the
+// scale e^{F_t + R_t} cancels in the readout ratio, and at the chunk's end it is the
+// new log-scale m' = F_{L-1} + R_{L-1}, which equals the token-by-token stabiliser.
+// Every exponent is <= 0.  The readout of row t (token u = t0 + t - D) is
+//   h = (e^{m-R_t} q~_u^T C + sum_s W_ts v~_s) / (e^{m-R_t} q~_u^T z + sum_s W_ts),
+//   W_ts = e^{g_s - R_t} (q~_u . k~_s)  for s <= t,
+// so a chunk costs three small dense products (q~ K^T, q~ C, W V) plus the state
+// update C' = e^{m - R_{L-1}} C + K^T diag(e^{g - R_{L-1}}) V, all from shared memory
+// with register tiles; chunks follow one another, the tokens of a chunk do not.
+constexpr int CL = 64;             // tokens per chunk
+
+template <int HD>
+struct ChunkLayout {
+  static constexpr int HH = HD / 2;
+  static constexpr int QS = HD + 4;              // row strides (floats), multiples of 4
+  static constexpr int VS = HH + 4;
+  static constexpr int WS = CL + 4;
+  static constexpr int OFF_Q = 0;                // [CL][QS]  q~ of the read-out tokens
+  static constexpr int OFF_K = OFF_Q + CL * QS;  // [CL][QS]  k~ of the chunk's tokens
+  static constexpr int OFF_V = OFF_K + CL * QS;  // [CL][VS]  v~
+  static constexpr int OFF_C = OFF_V + CL * VS;  // [HD][VS]  state C
+  static constexpr int OFF_W = OFF_C + HD * VS;  // [CL][WS]  W_ts
+  static constexpr int OFF_Z = OFF_W + CL * WS;  // [HD]
+  static constexpr int OFF_G = OFF_Z + HD;       // [CL] g_s
+  static constexpr int OFF_R = OFF_G + CL;       // [CL] R_t
+  static constexpr int OFF_QZ = OFF_R + CL;      // [CL] q~ . z
+  static constexpr int OFF_SC = OFF_QZ + CL;     // [4] m, F_{L-1}
+  static constexpr int FLOATS = OFF_SC + 4;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(NTM) mlstm_chunk_kernel(MScanArgs a) {
+  using Ly = ChunkLayout<HD>;
+  constexpr int HH = Ly::HH, QS = Ly::QS, VS = Ly::VS, WS = Ly::WS;
+  constexpr int NB = HH / 16;                    // column blocks of q~C / num per thread
   const Dims& dm = a.dm;
-  const int d = dm.d, D = dm.D, H = dm.H, hh = d / 2, NF = a.NF;
+  const int D = dm.D, H = dm.H, NF = a.NF;
   const int lp = blockIdx.x, bl = lp / H, h = lp - bl * H;
   const int pair = (a.first_seq + bl) * H + h;
   const int P = a.plen[bl];
   const size_t Pm = a.Pmax;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  extern __shared__ __align__(16) unsigned char smem[];
-  float* C = reinterpret_cast<float*>(smem);                   // [d][hh]
-  float* z = C + d * hh;                                        // [d]
-  float* ft = z + d;                                            // [NF] features of token t
-  float* qu = ft + NF;                                          // [d]  q~ of token u
-  float* red = qu + d;                                          // [NTM]
-  __shared__ float s_den, s_r;
-  for (int e = tid; e < d * hh; e += NTM) C[e] = 0.f;
-  for (int e = tid; e < d; e += NTM) z[e] = 0.f;
-  float m = -INFINITY;
+  const int ty = tid >> 4, tx = tid & 15;        // 16 x 16 thread grid
+  extern __shared__ __align__(16) float smf[];
+  float* Qs = smf + Ly::OFF_Q;
+  float* Ks = smf + Ly::OFF_K;
+  float* Vs = smf + Ly::OFF_V;
+  float* Cs = smf + Ly::OFF_C;
+  float* Ws = smf + Ly::OFF_W;
+  float* zs = smf + Ly::OFF_Z;
+  float* gs = smf + Ly::OFF_G;
+  float* Rs = smf + Ly::OFF_R;
+  float* qz = smf + Ly::OFF_QZ;
+  float* sc = smf + Ly::OFF_SC;
+  for (int e = tid; e < HD * VS; e += NTM) Cs[e] = 0.f;
+  for (int e = tid; e < HD; e += NTM) zs[e] = 0.f;
+  if (tid == 0) sc[0] = -INFINITY;
   const float* F = a.feat + (size_t)lp * Pm * NF;
   float* prio = a.prio + (size_t)lp * Pm;
-  const int groups = NTM / hh;                                  // row groups of the readout
-  const int jr = tid % hh, gr = tid / hh;
-  // features of the next token (and the next read-out query) are fetched into
-  // registers one iteration ahead; NF <= 2 * NTM and d <= NTM
-  float nf0 = 0.f, nf1 = 0.f, nq = 0.f;
-  auto fetch = [&](int t) {
-    if (t >= P) return;
-    nf0 = tid < NF ? F[(size_t)t * NF + tid] : 0.f;
-    nf1 = tid + NTM < NF ? F[(size_t)t * NF + tid + NTM] : 0.f;
-    nq = (t >= D && tid < d) ? F[(size_t)(t - D) * NF + d + hh + tid] : 0.f;
-  };
-  fetch(0);
-  for (int t = 0; t < P; ++t) {
-    __syncthreads();
-    if (tid < NF) ft[tid] = nf0;
-    if (tid + NTM < NF) ft[tid + NTM] = nf1;
-    if (t >= D && tid < d) qu[tid] = nq;
-    fetch(t + 1);
-    __syncthreads();    const float ai = ft[2 * d + hh], af = ft[2 * d + hh + 1];
-    const float lf = -softplus(-af);
-    const float m_new = fmaxf(lf + m, ai);
-    const float fs = (m == -INFINITY) ? 0.f : expf(lf + m - m_new);
-    const float is = expf(ai - m_new);
-    m = m_new;
-    for (int e = tid; e < d * hh; e += NTM) {
-      const int i = e / hh, j = e - i * hh;
-      C[e] = fmaf(fs, C[e], is * ft[i] * ft[d + j]);
-    }
-    for (int e = tid; e < d; e += NTM) z[e] = fmaf(fs, z[e], is * ft[e]);
-    if (t < D) continue;
-    __syncthreads();
-    // readout y_j = sum_i q~_i C[i][j], den = q~ . z
-    float y = 0.f;
-    if (gr < groups)
-      for (int i = gr; i < d; i += groups) y = fmaf(qu[i], C[i * hh + jr], y);
-    red[tid] = y;
-    if (warp == 0) {
-      float dd = 0.f;
-      for (int i = lane; i < d; i += 32) dd = fmaf(qu[i], z[i], dd);
-      dd = warp_sum(dd);
-      if (lane == 0) s_den = dd;
-    }
-    __syncthreads();
-    if (warp == 0) {
-      float rp = 0.f;
-      for (int j = lane; j < hh; j += 32) {
-        float yy = 0.f;
-        for (int g = 0; g < groups; ++g) yy += red[g * hh + j];
-        const float hv = yy / s_den;
-        rp = fmaf(a.ms.a[(size_t)h * hh + j], hv / (1.f + expf(-hv)), rp);
-      }
-      rp = warp_sum(rp);
-      if (lane == 0) {
-        const int u = t - D;
-        float r = rp + a.ms.b[h];
-        if (a.override_) r = a.override_[(size_t)lp * Pm + u];
-        prio[u] = static_priority(canon_score(r), u, a.st.log_gamma, h);
-      }
-    }
-  }
+  const float* av = a.ms.a + (size_t)h * HH;
+  const float bsc = a.ms.b[h];
   __syncthreads();
-  float* Cg = a.ms.C + (size_t)pair * d * hh;
-  for (int e = tid; e < d * hh; e += NTM) Cg[e] = C[e];
-  for (int e = tid; e < d; e += NTM) a.ms.z[(size_t)pair * d + e] = z[e];
-  if (tid == 0) a.ms.m[pair] = m;
+
+  for (int t0 = 0; t0 < P; t0 += CL) {
+    // ---- load the chunk: k~, v~ of tokens t0.., q~ of the tokens they read out ------
+    for (int e = tid; e < CL * (HD / 4); e += NTM) {
+      const int r = e / (HD / 4), c4 = e - r * (HD / 4);
+      const int t = t0 + r, u = t - D;
+      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), qv = kv;
+      if (t < P) kv = *reinterpret_cast<const float4*>(F + (size_t)t * NF + 4 * c4);
+      if (t < P && u >= 0) qv = *reinterpret_cast<const float4*>(F + (size_t)u * NF + HD + HH + 4 * c4);
+      *reinterpret_cast<float4*>(Ks + r * QS + 4 * c4) = kv;
+      *reinterpret_cast<float4*>(Qs + r * QS + 4 * c4) = qv;
+    }
+    for (int e = tid; e < CL * HH; e += NTM) {
+      const int r = e / HH, j = e - r * HH;
+      const int t = t0 + r;
+      Vs[r * VS + j] = t < P ? F[(size_t)t * NF + HD + j] : 0.f;
+    }
+    // gates: warp 0 scans the chunk's log forget gates (two tokens per lane)
+    if (warp == 0) {
+      const float m = sc[0];
+      float lfv[2], aiv[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int t = t0 + 2 * lane + k;
+        const bool in = t < P;
+        aiv[k] = in ? F[(size_t)t * NF + 2 * HD + HH] : -INFINITY;
+        lfv[k] = in ? -softplus(-F[(size_t)t * NF + 2 * HD + HH + 1]) : 0.f;
+      }
+      float f1 = lfv[0] + lfv[1], inc = f1;          // inclusive scan over lane pairs
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      const float Fa = inc - f1 + lfv[0], Fb = inc;  // F of tokens 2 lane, 2 lane + 1
+      const float ga = aiv[0] - Fa, gb = aiv[1] - Fb;
+      float gm = fmaxf(ga, gb), run = gm;            // inclusive prefix max
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, run, o);
+        if (lane >= o) run = fmaxf(run, y);
+      }
+      const float prev = __shfl_up_sync(0xffffffffu, run, 1);
+      const float before = lane == 0 ? -INFINITY : prev;
+      gs[2 * lane] = ga;
+      gs[2 * lane + 1] = gb;
+      Rs[2 * lane] = fmaxf(m, fmaxf(before, ga));
+      Rs[2 * lane + 1] = fmaxf(m, run);
+      if (lane == 31) sc[1] = Fb;                    // F of the chunk's last token
+      (void)gm;
+    }
+    __syncthreads();
+
+    // ---- S = q~ K^T -> W;  q~ C -> registers;  q~ . z ----------------------------------
+    {
+      float acc[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+      for (int c = 0; c < HD; c += 4) {
+        float4 qa[4], kb[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) qa[i] = *reinterpret_cast<const float4*>(Qs + (ty + 16 * i) * QS + c);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) kb[j] = *reinterpret_cast<const float4*>(Ks + (tx + 16 * j) * QS + c);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            acc[i][j] = fmaf(qa[i].x, kb[j].x, fmaf(qa[i].y, kb[j].y,
+                        fmaf(qa[i].z, kb[j].z, fmaf(qa[i].w, kb[j].w, acc[i][j]))));
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = ty + 16 * i;
+        const float R = Rs[t];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int s = tx + 16 * j;
+          Ws[t * WS + s] = (s <= t) ? __expf(gs[s] - R) * acc[i][j] : 0.f;
+        }
+      }
+    }
+    float num[4][NB];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < NB; ++j) num[i][j] = 0.f;
+#pragma unroll 2
+    for (int c = 0; c < HD; c += 4) {
+      float4 qa[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) qa[i] = *reinterpret_cast<const float4*>(Qs + (ty + 16 * i) * QS + c);
+#pragma unroll
+      for (int j = 0; j < NB; ++j) {
+        const int col = tx + 16 * j;
+        const float c0 = Cs[(c + 0) * VS + col], c1 = Cs[(c + 1) * VS + col];
+        const float c2 = Cs[(c + 2) * VS + col], c3 = Cs[(c + 3) * VS + col];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          num[i][j] = fmaf(qa[i].x, c0, fmaf(qa[i].y, c1, fmaf(qa[i].z, c2, fmaf(qa[i].w, c3, num[i][j]))));
+      }
+    }
+    // q~ . z: warp w takes rows 8w .. 8w + 7
+#pragma unroll
+    for (int rr = 0; rr < CL / 8; ++rr) {
+      const int t = warp * (CL / 8) + rr;
+      float s = 0.f;
+      for (int c = lane; c < HD; c += 32) s = fmaf(Qs[t * QS + c], zs[c], s);
+      s = warp_sum(s);
+      if (lane == 0) qz[t] = s;
+    }
+    __syncthreads();
+
+    // ---- readout rows: num = e^{m-R} q~C + W V, den = e^{m-R} q~.z + sum_s W ----------
+    {
+      const float m = sc[0];
+      float den[4], coef[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = ty + 16 * i;
+        coef[i] = __expf(m - Rs[t]);
+        den[i] = 0.f;
+#pragma unroll
+        for (int j = 0; j < NB; ++j) num[i][j] *= coef[i];
+      }
+#pragma unroll 4
+      for (int s = 0; s < CL; s += 4) {
+        float4 wa[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          wa[i] = *reinterpret_cast<const float4*>(Ws + (ty + 16 * i) * WS + s);
+          den[i] += (wa[i].x + wa[i].y) + (wa[i].z + wa[i].w);
+        }
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+          const int col = tx + 16 * j;
+          const float v0 = Vs[(s + 0) * VS + col], v1 = Vs[(s + 1) * VS + col];
+          const float v2 = Vs[(s + 2) * VS + col], v3 = Vs[(s + 3) * VS + col];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            num[i][j] = fmaf(wa[i].x, v0, fmaf(wa[i].y, v1, fmaf(wa[i].z, v2, fmaf(wa[i].w, v3, num[i][j]))));
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = ty + 16 * i;
+        const float dn = fmaf(coef[i], qz[t], den[i]);
+        float r = 0.f;
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+          const float hv = num[i][j] / dn;
+          r = fmaf(av[tx + 16 * j], hv / (1.f + expf(-hv)), r);
+        }
+#pragma unroll
+        for (int o = 1; o < 16; o <<= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+        const int T = t0 + t, u = T - D;
+        if (tx == 0 && T < P && u >= 0) {
+          float rv = r + bsc;
+          if (a.override_) rv = a.override_[(size_t)lp * Pm + u];
+          prio[u] = static_priority(canon_score(rv), u, a.st.log_gamma, h);
+        }
+      }
+    }
+    // ---- state update C' = e^{m-R_L} C + K^T diag(e^{g-R_L}) V;  z likewise -------------
+    {
+      const float RL = Rs[CL - 1];
+      const float wc = __expf(sc[0] - RL);
+      constexpr int NR = HD / 16;
+      float acc[NR][NB];
+#pragma unroll
+      for (int i = 0; i < NR; ++i)
+#pragma unroll
+        for (int j = 0; j < NB; ++j) acc[i][j] = wc * Cs[(ty + 16 * i) * VS + tx + 16 * j];
+#pragma unroll 4
+      for (int s = 0; s < CL; ++s) {
+        const float w = __expf(gs[s] - RL);
+        float vb[NB];
+#pragma unroll
+        for (int j = 0; j < NB; ++j) vb[j] = w * Vs[s * VS + tx + 16 * j];
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+          const float kk = Ks[s * QS + ty + 16 * i];
+#pragma unroll
+          for (int j = 0; j < NB; ++j) acc[i][j] = fmaf(kk, vb[j], acc[i][j]);
+        }
+      }
+      float zn = 0.f;
+      if (tid < HD) {
+        zn = wc * zs[tid];
+        for (int s = 0; s < CL; ++s) zn = fmaf(__expf(gs[s] - RL), Ks[s * QS + tid], zn);
+      }
+      __syncthreads();                 // every read of C, z and the scalars is done
+#pragma unroll
+      for (int i = 0; i < NR; ++i)
+#pragma unroll
+        for (int j = 0; j < NB; ++j) Cs[(ty + 16 * i) * VS + tx + 16 * j] = acc[i][j];
+      if (tid < HD) zs[tid] = zn;
+      if (tid == 0) sc[0] = sc[1] + RL;
+    }
+    __syncthreads();
+  }
+  float* Cg = a.ms.C + (size_t)pair * HD * HH;
+  for (int e = tid; e < HD * HH; e += NTM) Cg[e] = Cs[(e / HH) * VS + (e % HH)];
+  for (int e = tid; e < HD; e += NTM) a.ms.z[(size_t)pair * HD + e] = zs[e];
+  if (tid == 0) a.ms.m[pair] = sc[0];
 }
+
+template <int HD>
+size_t chunk_smem() { return (size_t)ChunkLayout<HD>::FLOATS * 4; }
 
 }  // namespace
 
@@ -471,6 +662,9 @@ cudaError_t prepare_mlstm(const Dims& dm) {
     if (e == cudaSuccess)
       e = raise_smem_limit(mlstm_proj_kernel<bf16>, psm);
   }
+  if (e == cudaSuccess)
+    e = dm.d == 128 ? raise_smem_limit(mlstm_chunk_kernel<128>, chunk_smem<128>())
+                    : raise_smem_limit(mlstm_chunk_kernel<64>, chunk_smem<64>());
   return e;
 }
 
@@ -517,8 +711,10 @@ cudaError_t launch_prefill_mlstm_scores(const State& st, const Dims& dm, const M
     if (e != cudaSuccess) return e;
   }
   MScanArgs sa{st, dm, to_mstate(m), plen, feat, override_, prio, first_seq, Pmax, NF};
-  const size_t ssm = ((size_t)dm.d * (dm.d / 2) + dm.d + NF + dm.d + NTM) * 4;
-  mlstm_scan_kernel<<<pairs, NTM, ssm, stream>>>(sa);
+  if (dm.d == 128)
+    mlstm_chunk_kernel<128><<<pairs, NTM, chunk_smem<128>(), stream>>>(sa);
+  else
+    mlstm_chunk_kernel<64><<<pairs, NTM, chunk_smem<64>(), stream>>>(sa);
   return cudaGetLastError();
 }
 

@@ -476,8 +476,10 @@ __global__ void __launch_bounds__(NT2) prefill_select_kernel(SelectArgs<T> a) {
   const unsigned char* Vp = reinterpret_cast<const unsigned char*>(a.V) + ((size_t)bl * H + h) * Pm * R;
   unsigned char* sK = static_cast<unsigned char*>(a.st.slotK) + (size_t)pair * B * R;
   unsigned char* sV = static_cast<unsigned char*>(a.st.slotV) + (size_t)pair * B * R;
-  for (int slot = warp; slot < nkept; slot += NT2 / 32) {
+  dcheck(nkept <= B, a.st.err, DEVERR_INDEX);
+  for (int slot = warp; slot < min(nkept, B); slot += NT2 / 32) {
     const int u = ps[slot];
+    if (!dcheck(u >= 0 && u < P, a.st.err, DEVERR_INDEX)) continue;
     for (int c = lane; c < chunks; c += 32) {
       reinterpret_cast<uint4*>(sK + (size_t)slot * R)[c] =
           reinterpret_cast<const uint4*>(Kp + (size_t)u * R)[c];

@@ -30,13 +30,15 @@ __device__ __forceinline__ long long cta_begin(long long c, long long T, long lo
 // __syncthreads; every thread of the block must call it.
 template <int NT>
 __device__ __forceinline__ void build_schedule(const int32_t* __restrict__ nvalid,
-                                               const int32_t* __restrict__ len, int npairs,
-                                               int D, int tile, int* prefix, int* scan) {
+                                               const int32_t* __restrict__ len, int npairs, int B,
+                                               int D, int tile, int* prefix, int* scan,
+                                               int32_t* err) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int per = (npairs + NT - 1) / NT;
   const int beg = min(tid * per, npairs), end = min(beg + per, npairs);
   int local = 0;
-  for (int i = beg; i < end; ++i) local += tiles_of(nvalid[i], min(len[i], D), tile);
+  for (int i = beg; i < end; ++i)
+    local += tiles_of(used_slots(nvalid[i], B, err), window_rows(len[i], D, err), tile);
   int incl = local;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
@@ -54,7 +56,7 @@ __device__ __forceinline__ void build_schedule(const int32_t* __restrict__ nvali
   int run = scan[warp] + incl - local;
   for (int i = beg; i < end; ++i) {
     prefix[i] = run;
-    run += tiles_of(nvalid[i], min(len[i], D), tile);
+    run += tiles_of(used_slots(nvalid[i], B, nullptr), window_rows(len[i], D, nullptr), tile);
   }
   __syncthreads();
 }

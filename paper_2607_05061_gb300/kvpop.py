@@ -16,7 +16,10 @@ from typing import Optional, Sequence
 import torch  # loads the CUDA runtime the library links against
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libkvpop.so")
+# KVPOP_DEVICE_CHECKS=1 selects the device-check build (index checks that record an
+# error instead of trapping), built by ``build.build(checked=True)``
+CHECKED = os.environ.get("KVPOP_DEVICE_CHECKS", "0") == "1"
+LIB_PATH = os.path.join(_HERE, "libkvpop_checked.so" if CHECKED else "libkvpop.so")
 
 KVPOP_F32, KVPOP_BF16 = 0, 1
 STATUS = {0: "KVPOP_OK", 1: "KVPOP_ERR_INVALID_ARG", 2: "KVPOP_ERR_ALIGN", 3: "KVPOP_ERR_OOM",
@@ -24,6 +27,7 @@ STATUS = {0: "KVPOP_OK", 1: "KVPOP_ERR_INVALID_ARG", 2: "KVPOP_ERR_ALIGN", 3: "K
 
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2607_05061_gb300.build`"
+                      + (" -c" if CHECKED else "") +
                       " (or __graft_entry__.build()); the decode path has no non-CUDA fallback")
 _lib = ctypes.CDLL(LIB_PATH)
 
@@ -84,6 +88,7 @@ _SIGS = {
     "kvpop_standalone_status": (ctypes.c_int, [_P]),
     "kvpop_last_error": (ctypes.c_char_p, []),
     "kvpop_debug_fail_alloc_after": (None, [c_int32]),
+    "kvpop_debug_skip_attention_copies": (None, [c_int32]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _name)
