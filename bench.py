@@ -637,7 +637,7 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
     attn_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
     # end to end: host hidden state in (pinned), final hidden state out, per step
     E = max(1, min(args.e2e_steps, 64))
-    xh = xs[:E].cpu().pin_memory()
+    xh = gen.decode_hidden(cfg, L, W + K + n_attn, E).pin_memory()
     oh = torch.empty((cfg.batch, cfg.hidden), dtype=torch.bfloat16).pin_memory()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
