@@ -383,9 +383,9 @@ def run_kvpop(args):
     q, k, v = gen.decode_inputs(cfg, L, 0, W + K + post + 2, device=dev)
     out = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
+    fused = cache.fused_step           # one kernel per kvpop_decode_step
     for j in range(W):
-        cache.ingest(q[j], k[j], v[j])
-        cache.attend(q[j], out)
+        cache.step(q[j], k[j], v[j], out)
     torch.cuda.synchronize()
 
     def ev():
@@ -413,8 +413,7 @@ def run_kvpop(args):
     if not flush:
         def timed_body():
             for i in range(K):
-                cache.ingest(q[W + i], k[W + i], v[W + i])
-                cache.attend(q[W + i], out)
+                cache.step(q[W + i], k[W + i], v[W + i], out)
         graph = capture(timed_body)
     clocks = ClockSampler(local_rank)
     clocks.start()
@@ -426,8 +425,7 @@ def run_kvpop(args):
         for i in range(K):
             flush_buf.fill_(float(i))
             step_ev[i][0].record(stream)
-            cache.ingest(q[W + i], k[W + i], v[W + i])
-            cache.attend(q[W + i], out)
+            cache.step(q[W + i], k[W + i], v[W + i], out)
             step_ev[i][1].record(stream)
     else:
         graph.replay()
@@ -442,29 +440,38 @@ def run_kvpop(args):
     else:
         step_ms_local = t_start.elapsed_time(t_end) / K
     del graph
-    # The attention kernel's own duration: ATTN_POST_LAUNCHES further decode steps with
-    # events around each attention (events between the ingest and the attention stop the
-    # attention from launching as a programmatic dependent of the ingest, which is why
-    # the timed steps carry none); the first two, which wait for the host to enqueue
-    # them after the synchronisation, are not counted.
+    # The dominant kernel's own duration: ATTN_POST_LAUNCHES further decode steps with
+    # events around each launch of it -- the whole step where it is one kernel, else the
+    # attention (events between the ingest and the attention stop the attention from
+    # launching as a programmatic dependent of the ingest, which is why the timed steps
+    # carry none); the first two, which wait for the host to enqueue them after the
+    # synchronisation, are not counted.
     attn_ev = []
     for i in range(post + 2):
         j = W + K + i
-        cache.ingest(q[j], k[j], v[j])
+        if not fused:
+            cache.ingest(q[j], k[j], v[j])
         if flush:
             flush_buf.fill_(float(i))
         a, b = ev(), ev()
         a.record(stream)
-        cache.attend(q[j], out)
+        if fused:
+            cache.step(q[j], k[j], v[j], out)
+        else:
+            cache.attend(q[j], out)
         b.record(stream)
         attn_ev.append((a, b))
     torch.cuda.synchronize()
     cache.check()
     attn_ms = statistics.mean(a.elapsed_time(b) for a, b in attn_ev[2:])
     attn_bytes = mean_stream_bytes(cfg, L, W + K + 2, post)
-    attn_how = (f"CUDA events around the attention in {post} decode steps after the timed "
-                f"region (the ingest between them untimed" +
-                (", L2 flushed before each)" if flush else ")"))
+    if fused:
+        attn_how = (f"CUDA events around each of {post} one-kernel decode steps after the timed "
+                    f"region" + (", L2 flushed before each" if flush else ""))
+    else:
+        attn_how = (f"CUDA events around the attention in {post} decode steps after the timed "
+                    f"region (the ingest between them untimed" +
+                    (", L2 flushed before each)" if flush else ")"))
 
     # end to end through the C ABI on host buffers (pinned), copies inside the timed region
     E = max(1, args.e2e_steps)
@@ -531,7 +538,8 @@ def run_kvpop(args):
         "steps_per_s": 1e3 / step_ms,
         "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
         "prefill_s": t_prefill,
-        "roofline": {"bound": "hbm", "kernel": ("attend_tc_kernel" if cfg.kv_dtype == "bf16"
+        "roofline": {"bound": "hbm", "kernel": ("attend_tc_kernel<fused step>" if fused else
+                                                 "attend_tc_kernel" if cfg.kv_dtype == "bf16"
                                                  else "attend_kernel"),
                      "achieved": achieved, "peak": peak,
                      "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
@@ -545,7 +553,7 @@ def run_kvpop(args):
                 "how": "kvpop_decode_step_host on pinned host buffers (q|k|v packed: one copy in; "
                        "the attention writes out into pinned host memory), stream sync every step"
                        + ("; L2 flushed before each step, outside its timing" if flush else "")},
-        "gpu_launches": 2 * K,
+        "gpu_launches": K if fused else 2 * K,
         "clocks": clk,
     }
     cache.free()
@@ -614,7 +622,9 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
     for c in st.caches:
         c.check()
     step_ms_local = t_start.elapsed_time(t_end) / K
-    # attention launch durations: eager steps with events around every layer's attention
+    # durations of the dominant kernel: eager steps with events around every layer's
+    # one-kernel decode step (or, on the two-kernel path, around its attention)
+    fused = all(c.fused_step for c in st.caches)
     ev = []
     x = torch.empty_like(x_in)
     for i in range(n_attn):
@@ -623,10 +633,14 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
             torch.matmul(xcur, Lw["Wq"], out=st.q)
             torch.matmul(xcur, Lw["Wk"], out=st.k)
             torch.matmul(xcur, Lw["Wv"], out=st.v)
-            cache.ingest(st.q, st.k, st.v)
+            if not fused:
+                cache.ingest(st.q, st.k, st.v)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            cache.attend(st.q, st.o)
+            if fused:
+                cache.step(st.q, st.k, st.v, st.o)
+            else:
+                cache.attend(st.q, st.o)
             e1.record(stream)
             ev.append((e0, e1))
             st.o_bf.copy_(st.o)
@@ -671,7 +685,8 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "steps_per_s": 1e3 / step_ms,
         "hbm_gbs_step": (cfg.n_layers * bytes_per_launch + proj_bytes) / (step_ms / 1e3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": "attend_tc_kernel", "achieved": achieved, "peak": peak,
+        "roofline": {"bound": "hbm", "kernel": "attend_tc_kernel<fused step>" if fused else "attend_tc_kernel",
+                     "achieved": achieved, "peak": peak,
                      "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)", "unit": "GB/s",
                      "frac": achieved / peak, "frac_of_8tbs_nominal": achieved / 8000.0,
                      "traffic": None, "algorithmic_bytes_per_launch": bytes_per_launch,
@@ -680,7 +695,7 @@ def run_stack_bench(args, cfg, rank, local_rank, world, dev, dist):
                 "h2d_bytes_per_step": cfg.batch * cfg.hidden * 2,
                 "d2h_bytes_per_step": cfg.batch * cfg.hidden * 2, "steps": E,
                 "how": "pinned hidden state in, graph replay, final hidden state out, sync per step"},
-        "gpu_launches": K * cfg.n_layers * 2,
+        "gpu_launches": K * cfg.n_layers * (1 if fused else 2),
         "clocks": clk,
         "cpu_baseline": None,
         "cpu_baseline_note": ("not run for the stack: the fp64 oracle would have to prefill 36 layers "

@@ -295,11 +295,28 @@ kvpop_status kvpop_decode_ingest(kvpop_cache* cache, const void* q_dev, const vo
 kvpop_status kvpop_decode_attend(kvpop_cache* cache, const void* q_dev, float* out_dev,
                                  cudaStream_t stream);
 
-/* kvpop_decode_ingest followed by kvpop_decode_attend. */
+/* One whole decode step (Sec. 3.1-3.3, App. C): the effect of kvpop_decode_ingest
+ * followed by kvpop_decode_attend, with the same arguments and outputs.  For bf16
+ * caches with d = 128, a scorer hidden width F <= 256, up to about 2000 (sequence,
+ * KV head) pairs, and a K/V stream of at least 600 MB per step at full budget
+ * (pairs x (B + D) x 2 d x 2 bytes; below that the scorer would outlast the
+ * attention) it runs as one kernel: the attention streams every key that cannot change in this
+ * step while the scorer, keep-or-drop and scatter run beside it, and the one slot and
+ * the one window row that may change are added when each (sequence, KV head) is
+ * merged (kvpop_step_is_fused reports 1).  The attention output may then differ from
+ * the two-call path by the order of its fp32 sums; evictions follow the same rule.
+ * The environment variables KVPOP_SPLIT_STEP / KVPOP_FUSED_STEP, set before
+ * kvpop_init_cache, choose the two-kernel / one-kernel path regardless of the stream
+ * size (the shape and shared-memory conditions still apply).  Asynchronous on
+ * `stream`. */
 kvpop_status kvpop_decode_step(kvpop_cache* cache, const void* q_dev, const void* k_dev,
                                const void* v_dev, float* out_dev,
                                const float* score_override_dev, int32_t* evict_info_dev,
                                float* score_out_dev, cudaStream_t stream);
+
+/* 1 when kvpop_decode_step of this cache runs as one kernel, 0 when it runs the
+ * ingest and the attention as two, -1 for an invalid handle. */
+int32_t kvpop_step_is_fused(const kvpop_cache* cache);
 
 /* kvpop_decode_step on host buffers (pinned memory recommended): copies q/k/v
  * into library-owned device staging (one copy when k_host and v_host follow q_host

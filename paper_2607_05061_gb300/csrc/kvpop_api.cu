@@ -27,6 +27,9 @@ struct kvpop_cache {
   std::vector<void*> allocs;
   std::vector<unsigned char> tc_maps;   // TMA descriptors of the K/V stores (bf16 path)
   bool use_tc = false;
+  bool use_fused = false;               // kvpop_decode_step as one kernel (bf16, d = 128)
+  FusedBufs fb{};
+  int fused_grid = 0;
   bool use_cluster = false;             // cluster ingest kernel
   float* W1s = nullptr;                 // slice-major scorer weights for it
   float* b1s = nullptr;
@@ -63,6 +66,9 @@ namespace {
 int32_t* standalone_err() { return kvpop::standalone_err_word(); }
 
 constexpr uint64_t kMagic = 0x6b7670'6f70'6361ull;   // "kvpopca"
+// K/V bytes per step from which kvpop_decode_step runs as one kernel: the attention then
+// takes at least ~90 us, about what the scorer units need beside it on the GPU.
+constexpr double kFusedMinStepBytes = 600e6;
 constexpr uint64_t kStateVersion = 1;
 int g_fail_after = 0;
 thread_local char g_last_error[256] = "";
@@ -304,7 +310,34 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     if (s == KVPOP_OK && occ < 1) s = KVPOP_ERR_INVALID_ARG;
     c->attend_grid = sms * (occ > 0 ? occ : 1);
   }
-  ALLOC(part, float*, (size_t)2 * c->attend_grid * (dm.G * d + 2 * dm.G) * 4)
+  // the one-kernel decode step, where its shape and shared memory allow it and the K/V
+  // stream of a step is long enough to hide the scorer behind it (otherwise
+  // kvpop_decode_step runs the ingest and the attention as two kernels)
+  AttendConfig fc;
+  const double step_kv_bytes = (double)pairs * (double)(B + D) * 2.0 * (double)d * (double)c->esz;
+  const bool want_fused = std::getenv("KVPOP_SPLIT_STEP") == nullptr &&
+                          (std::getenv("KVPOP_FUSED_STEP") != nullptr || step_kv_bytes >= kFusedMinStepBytes);
+  if (s == KVPOP_OK && c->use_tc && !c->mlstm && want_fused && tc_fused_ok(dm) &&
+      tc_fused_config(dm, &fc) == cudaSuccess) {
+    const size_t smem = fc.smem_fixed + (pairs + 1) * 4;
+    int occ_f = 0;
+    if (raise_smem_limit(fc.func, smem) == cudaSuccess &&
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ_f, fc.func, fc.threads, smem) == cudaSuccess &&
+        occ_f >= 1 && sms * occ_f <= tc_fused_max_grid()) {
+      c->use_fused = true;
+      c->fused_grid = sms * occ_f;
+    }
+    cudaGetLastError();   // a refused shared-memory size only disables the fused step
+  }
+  const size_t part_grid = c->fused_grid > c->attend_grid ? c->fused_grid : c->attend_grid;
+  ALLOC(part, float*, (size_t)2 * part_grid * (dm.G * d + 2 * dm.G) * 4)
+  if (s == KVPOP_OK && c->use_fused) {
+    s = dev_alloc(c, &p, pairs * (dm.G * d + 2 * dm.G) * 4);
+    c->fb.part_c = static_cast<float*>(p);
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * 4 * 4); c->fb.meta_next = (int32_t*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * (2 * dm.G + 2 * d) * 4); c->fb.xtra = (float*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, 16); c->fb.ctr = (int32_t*)p; }
+  }
 #undef ALLOC
   // q | k | v staging in one block, so that adjacent host buffers take a single copy
   if (s == KVPOP_OK) {
@@ -368,6 +401,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
       e = NOTE(cudaMemcpy2DAsync(w2, Fp * 4, sc->w2, F * 4, F * 4, H, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && sc) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && c->use_tf32) e = NOTE(prepare_score_tf32(dm, W1, c->w1t, sc_map_ptr(c), stream));
+    if (e == cudaSuccess && c->use_fused) e = NOTE(cudaMemsetAsync(c->fb.ctr, 0, 16, stream));
     std::vector<float> minus_inf;
     if (c->mlstm) {
       // mLSTM weights: column blocks of Wcat [2d][NC] = [W_k | W_v | W_q | w_i | w_f | 0]
@@ -708,9 +742,23 @@ kvpop_status kvpop_decode_step(kvpop_cache* c, const void* q, const void* k, con
   if (s != KVPOP_OK) return s;
   if (!out) return KVPOP_ERR_INVALID_ARG;
   if (!aligned16(out)) return KVPOP_ERR_ALIGN;
+  if (c->use_fused) {
+    if (!q || !k || !v) return KVPOP_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned4(override_) ||
+        !aligned4(evict_info) || !aligned4(score_out))
+      return KVPOP_ERR_ALIGN;
+    return poison_on(c, NOTE(tc_launch_fused(c->st, c->dm, tc_map_ptr(c), c->fb, q, k, v, out,
+                                             override_, evict_info, score_out, c->fused_grid,
+                                             stream)));
+  }
   s = kvpop_decode_ingest(c, q, k, v, override_, evict_info, score_out, stream);
   if (s != KVPOP_OK) return s;
   return kvpop_decode_attend(c, q, out, stream);
+}
+
+int32_t kvpop_step_is_fused(const kvpop_cache* c) {
+  if (!c || c->magic != kMagic) return -1;
+  return c->use_fused ? 1 : 0;
 }
 
 kvpop_status kvpop_decode_step_host(kvpop_cache* c, const void* q, const void* k, const void* v,

@@ -21,8 +21,12 @@
 // and skips the remaining work while keeping every block barrier balanced.
 #include <cuda.h>
 
+#include <algorithm>
+#include <cstring>
+
 #include "kvpop_ptx.cuh"
 #include "kvpop_sched.cuh"
+#include "kvpop_step_fused.cuh"
 
 namespace kvpop {
 namespace {
@@ -40,6 +44,10 @@ constexpr float kThr = 8.0f;
 #ifndef KVPOP_TC_MINBLOCKS
 #define KVPOP_TC_MINBLOCKS 1
 #endif
+// Fused step: tiles (in 64ths) that a CTA with one scorer unit more than the rest gives up.
+#ifndef KVPOP_FUSED_SPLIT_K
+#define KVPOP_FUSED_SPLIT_K 5
+#endif
 
 template <int HD, int G>
 struct TcTraits {
@@ -50,6 +58,7 @@ struct TcTraits {
   static constexpr int TILE = 16 * NWC;
   static constexpr int STAGES = KVPOP_TC_STAGES;
   static constexpr int THREADS = (NWC + 1) * 32;
+  static constexpr int THREADS_F = (NWC + 1 + kFusedSW) * 32;   // with the scorer warps
   static constexpr int HALF_BYTES = TILE * 128;    // one box
   static constexpr int STAGE_BYTES = 2 * NH * HALF_BYTES;
   static constexpr int al16(int x) { return (x + 15) & ~15; }
@@ -123,14 +132,19 @@ __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" ::"r"(KVPOP_TC_NWC * 32) : "memory");
 }
 
-template <int HD, int G>
-__global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
+// FUSED: the whole decode step (kvpop_step_fused.cuh): the consumers stream only the keys
+// that cannot change this step, the scorer warps ingest the new token meanwhile, and each
+// pair's last arrival merges.  Otherwise the attention alone, over the state the ingest left.
+template <int HD, int G, bool FUSED>
+__global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<HD, G>::THREADS,
+                                  KVPOP_TC_MINBLOCKS)
     attend_tc_kernel(const __grid_constant__ CUtensorMap mapSK, const __grid_constant__ CUtensorMap mapSV,
                      const __grid_constant__ CUtensorMap mapRK, const __grid_constant__ CUtensorMap mapRV,
-                     TcArgs a) {
+                     TcArgs a, const __grid_constant__ FusedArgs f) {
   using Tr = TcTraits<HD, G>;
   constexpr int TILE = Tr::TILE, NH = Tr::NH, NKS = Tr::NKS, NMT = Tr::NMT;
-  constexpr int STAGES = Tr::STAGES, NWC = Tr::NWC, NT = Tr::THREADS;
+  constexpr int STAGES = Tr::STAGES, NWC = Tr::NWC;
+  constexpr int NT = FUSED ? Tr::THREADS_F : Tr::THREADS;
 
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -152,21 +166,50 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     }
     mbar_fence_init();
   }
-  // Launched as a programmatic dependent of the ingest: everything below reads the
-  // state it writes, so wait here for it to complete (a no-op without a predecessor).
+  if constexpr (FUSED) {
+    // the next step's kernel may be scheduled now: it waits for this grid before reading
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  }
+  // Launched as a programmatic dependent of the kernel before it (the ingest, or the
+  // previous fused step): everything below reads the state it writes, so wait here for
+  // it to complete (a no-op without a predecessor).
   asm volatile("griddepcontrol.wait;" ::: "memory");
   build_schedule<NT>(a.nvalid, a.len, npairs, a.B, a.D, TILE, prefix, scan, a.err);
   const long long Ttot = prefix[npairs];
-  if (Ttot <= 0) return;
+  if constexpr (FUSED) {
+    // lengths and used-slot counts read: their commits may start once every CTA is here
+    if (tid == 0) {
+      __threadfence();
+      atomicAdd(f.ctr, 1);
+    }
+  } else {
+    if (Ttot <= 0) return;
+  }
   const long long NC = min((long long)gridDim.x, Ttot);
-  for (int p = blockIdx.x; p < npairs; p += gridDim.x)
-    if (prefix[p + 1] == prefix[p])
-      for (int i = tid; i < G * HD; i += NT) a.out[(size_t)p * G * HD + i] = 0.f;
-  if (blockIdx.x >= NC) return;
-  const long long t0 = cta_begin(blockIdx.x, Ttot, NC);
-  const long long t1 = cta_begin(blockIdx.x + 1, Ttot, NC);
-  int p0;
-  {
+  if constexpr (!FUSED) {
+    for (int p = blockIdx.x; p < npairs; p += gridDim.x)
+      if (prefix[p + 1] == prefix[p])
+        for (int i = tid; i < G * HD; i += NT) a.out[(size_t)p * G * HD + i] = 0.f;
+    if (blockIdx.x >= NC) return;
+  }
+  // FUSED: a CTA without tiles (or a step without any) still runs its scorer units, and
+  // the CTAs with one scorer unit more than the rest stream 3/64 fewer tiles (when every
+  // CTA has at least 4)
+  int* bnd = reinterpret_cast<int*>(smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::BND);
+  Split sp{Ttot, NC, bnd};
+  if constexpr (FUSED) {
+    const int units = f.H * ((f.batch + kFusedSeqs - 1) / kFusedSeqs);
+    const int extra = units % (int)gridDim.x;
+    const bool weigh = Ttot >= 4 * NC && extra > 0;
+    split_bounds(bnd, Ttot, NC, weigh ? (int)min((long long)extra, NC) : 0, weigh ? KVPOP_FUSED_SPLIT_K : 0,
+                 tid, NT);
+    __syncthreads();
+  }
+  const bool streams = Ttot > 0 && blockIdx.x < NC;
+  const long long t0 = streams ? (FUSED ? sp.begin(blockIdx.x) : cta_begin(blockIdx.x, Ttot, NC)) : 0;
+  const long long t1 = streams ? (FUSED ? sp.begin(blockIdx.x + 1) : cta_begin(blockIdx.x + 1, Ttot, NC)) : 0;
+  int p0 = 0;
+  if (streams) {
     int lo = 0, hi = npairs - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
@@ -174,12 +217,19 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     }
     p0 = lo;
   }
+  if constexpr (FUSED) {
+    if (warp > NWC) {
+      unsigned char* fsm = smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4);
+      fused_scorer<HD, G>(f, a.q, a.out, a.part, a.part_count, prefix, sp, a.D, a.B, a.qscale, fsm,
+                          tid - (NWC + 1) * 32);
+    }
+  }
 
   // ---- producer -------------------------------------------------------------------
   // With the testing hook on, the producer neither arms a barrier nor issues a copy:
   // every consumer's first bounded wait runs out, records DEVERR_TIMEOUT_FULL and the
   // consumers skip the rest of their work; no copy is in flight when the CTA exits.
-  if (warp == NWC) {
+  if (warp == NWC && streams) {
     if (lane == 0 && !a.skip_copies) {
       int p = p0;
       long long i = 0;
@@ -218,8 +268,9 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
                        DEVERR_TIMEOUT_DRAIN))
           break;
     }
-    return;
+    if constexpr (!FUSED) return;
   }
+  if (warp < NWC && streams) {
 
   // ---- consumers ------------------------------------------------------------------
   const int g8 = lane >> 2, t4 = lane & 3;            // fragment row group / column pair
@@ -228,8 +279,17 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
   float m0, m1, l0, l1;                                // heads 2*t4, 2*t4 + 1
   bool ok = true;
   int cur = -1;
+  // FUSED: the slot that may change this step (full cache: the cached argmin) and the
+  // window row of the token leaving the window; both masked, merged by the last arrival
+  int cfull = -1, wmask = -1;
 
   auto load_q = [&](int p) {
+    if constexpr (FUSED) {
+      const int plen = a.len[p];
+      const int nvp = used_slots(a.nvalid[p], a.B, nullptr);
+      cfull = (plen >= a.D && nvp >= a.B) ? f.st.min_slot[p] : -1;
+      wmask = (plen >= a.D) ? plen % a.D : -1;
+    }
     const bf16* qp = a.q + ((size_t)p * G + g8) * HD;
 #pragma unroll
     for (int ks = 0; ks < NKS; ++ks) {
@@ -274,8 +334,63 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
       if (g8 == 0) { ml[warp * G + h1] = l1; mm[warp * G + h1] = m1; }
     }
     consumer_sync();
-    finish_pair<G, HD, NWC, NWC * 32>(p, prefix, Ttot, NC, t0, mo, ml, mm, a.out, a.part,
-                                      a.part_count, flag, [] { consumer_sync(); });
+    if constexpr (!FUSED) {
+      finish_pair<G, HD, NWC, NWC * 32>(p, prefix, Ttot, NC, t0, mo, ml, mm, a.out, a.part,
+                                        a.part_count, flag, [] { consumer_sync(); });
+    } else {
+      constexpr int NCT = NWC * 32, PSTRIDE = G * HD + 2 * G;
+      constexpr int EPT = MergeShape<HD, G, NCT>::EPT;
+      float om[EPT], ol[EPT], oo[EPT];
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) {
+        const int idx = tid + k * NCT;
+        om[k] = -INFINITY; ol[k] = 0.f; oo[k] = 0.f;
+        if (idx >= G * HD) continue;
+        const int g = idx / HD, i = idx - g * HD;
+        float ms = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NWC; ++w) ms = fmaxf(ms, mm[w * G + g]);
+        float L = 0.f, O = 0.f;
+#pragma unroll
+        for (int w = 0; w < NWC; ++w) {
+          const float mw = mm[w * G + g];
+          const float fw = (mw == -INFINITY) ? 0.f : exp2f(mw - ms);
+          L = fmaf(ml[w * G + g], fw, L);
+          O = fmaf(mo[(w * G + g) * HD + i], fw, O);
+        }
+        om[k] = ms; ol[k] = L; oo[k] = O;
+      }
+      long long ca, cb;
+      const int nctas = pair_ctas(p, prefix, sp, ca, cb);
+      // every other arrival (the other CTAs and the scorer) already in: merge from here
+      // without publishing this CTA's partial
+      if (tid == 0) *flag = (ld_acquire_gpu(a.part_count + p) == nctas);
+      consumer_sync();
+      bool last = *flag != 0;
+      if (!last) {
+        float* dst = (nctas == 1) ? f.part_c + (size_t)p * PSTRIDE
+                                  : a.part + ((size_t)blockIdx.x * 2 + ((prefix[p] < t0) ? 0 : 1)) * PSTRIDE;
+#pragma unroll
+        for (int k = 0; k < EPT; ++k) {
+          const int idx = tid + k * NCT;
+          if (idx >= G * HD) continue;
+          const int g = idx / HD, i = idx - g * HD;
+          dst[g * HD + i] = oo[k];
+          if (i == 0) { dst[G * HD + g] = om[k]; dst[G * HD + G + g] = ol[k]; }
+        }
+        __threadfence();
+        consumer_sync();
+        if (tid == 0) *flag = (atomicAdd(a.part_count + p, 1) == nctas);
+        consumer_sync();
+        last = *flag != 0;
+      }
+      if (last) {
+        __threadfence();
+        fused_merge<HD, G, NCT>(f, a.out, a.part, a.part_count, p, prefix, sp, (long long)blockIdx.x,
+                                om, ol, oo, tid, [] { consumer_sync(); });
+      }
+      consumer_sync();
+    }
   };
 
   const float qs = a.qscale;
@@ -295,7 +410,13 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     const int nvt = (nv + TILE - 1) / TILE;
     const int cnt = lt < nvt ? min(TILE, nv - lt * TILE)
                              : min(TILE, window_rows(a.len[p], a.D, nullptr) - (lt - nvt) * TILE);
-    dcheck(cnt > 0 && cnt <= TILE, a.err, DEVERR_INDEX);
+    if constexpr (!FUSED) dcheck(cnt > 0 && cnt <= TILE, a.err, DEVERR_INDEX);
+    int mrow = -1;                                     // FUSED: masked row of this tile
+    if constexpr (FUSED) {
+      const int r = (lt < nvt) ? (cfull >= 0 ? cfull - lt * TILE : -1)
+                               : (wmask >= 0 ? wmask - (lt - nvt) * TILE : -1);
+      mrow = (r >= 0 && r < TILE) ? r : -1;
+    }
     const int key0 = warp * 16;
     if (ok && key0 < cnt) {
       const uint32_t kbase = smem_u32(smem + (size_t)s * Tr::STAGE_BYTES);
@@ -316,7 +437,8 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
           else        mma_bf16(c0, x0, x1, x2, x3, qb[ks][0], qb[ks][1]);
         }
       }
-      const bool va = key0 + g8 < cnt, vb = key0 + g8 + 8 < cnt;
+      const bool va = key0 + g8 < cnt && key0 + g8 != mrow;
+      const bool vb = key0 + g8 + 8 < cnt && key0 + g8 + 8 != mrow;
       float s0 = va ? (c0[0] + c1[0]) * qs : -INFINITY;   // key g8,   head 2 t4
       float s1 = va ? (c0[1] + c1[1]) * qs : -INFINITY;   // key g8,   head 2 t4 + 1
       float s2 = vb ? (c0[2] + c1[2]) * qs : -INFINITY;   // key g8+8, head 2 t4
@@ -374,6 +496,18 @@ __global__ void __launch_bounds__(TcTraits<HD, G>::THREADS, KVPOP_TC_MINBLOCKS)
     if (lane == 0) mbar_arrive(smem_u32(&bars[STAGES + s]));
   }
   if (cur >= 0) finalize(cur);
+  }   // consumers
+  if constexpr (FUSED) {
+    // the last CTA out re-arms the grid counters for the next step
+    __syncthreads();
+    if (tid == 0) {
+      __threadfence();
+      if (atomicAdd(f.ctr + 1, 1) == (int)gridDim.x - 1) {
+        f.ctr[0] = 0;
+        f.ctr[1] = 0;
+      }
+    }
+  }
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -435,6 +569,7 @@ cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out) {
 size_t tc_maps_size() { return sizeof(TcMaps); }
 
 #define TC_CASES(X) X(64, 1) X(64, 2) X(64, 4) X(128, 1) X(128, 2) X(128, 4)
+#define TC_FUSED_CASES(X) X(128, 1) X(128, 2) X(128, 4)
 
 cudaError_t tc_config(const Dims& dm, AttendConfig* out) {
 #define CFG(HD_, G_)                                                   \
@@ -442,7 +577,7 @@ cudaError_t tc_config(const Dims& dm, AttendConfig* out) {
     out->threads = TcTraits<HD_, G_>::THREADS;                         \
     out->smem_fixed = tc_smem<HD_, G_>(0) - 4;                         \
     out->tile = TcTraits<HD_, G_>::TILE;                               \
-    out->func = (const void*)attend_tc_kernel<HD_, G_>;                \
+    out->func = (const void*)attend_tc_kernel<HD_, G_, false>;         \
     return cudaSuccess;                                                \
   }
   TC_CASES(CFG)
@@ -450,9 +585,33 @@ cudaError_t tc_config(const Dims& dm, AttendConfig* out) {
   return cudaErrorInvalidValue;
 }
 
-cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const void* q, float* out,
-                      int grid, cudaStream_t stream) {
-  const TcMaps* m = static_cast<const TcMaps*>(maps);
+int tc_fused_max_grid() { return kMaxSplit; }
+
+bool tc_fused_ok(const Dims& dm) {
+  return dm.dtype == KVPOP_BF16 && dm.d == 128 && (dm.G == 1 || dm.G == 2 || dm.G == 4) &&
+         dm.F <= 256;
+}
+
+// Smem of the fused kernel: the attention's, then the scorer region after the prefix.
+static size_t tc_fused_smem_of(size_t attn_smem_pairs, int Fp) {
+  return ((attn_smem_pairs + 15) & ~size_t(15)) + fused_smem_bytes(Fp);
+}
+
+cudaError_t tc_fused_config(const Dims& dm, AttendConfig* out) {
+#define CFG(HD_, G_)                                                           \
+  if (dm.d == HD_ && dm.G == G_) {                                             \
+    out->threads = TcTraits<HD_, G_>::THREADS_F;                               \
+    out->smem_fixed = tc_fused_smem_of(tc_smem<HD_, G_>(0) - 4, dm.Fp) + 16;   \
+    out->tile = TcTraits<HD_, G_>::TILE;                                       \
+    out->func = (const void*)attend_tc_kernel<HD_, G_, true>;                  \
+    return cudaSuccess;                                                        \
+  }
+  if (tc_fused_ok(dm)) { TC_FUSED_CASES(CFG) }
+#undef CFG
+  return cudaErrorInvalidValue;
+}
+
+static TcArgs tc_args(const State& st, const Dims& dm, const void* q, float* out) {
   TcArgs a;
   a.nvalid = st.nvalid;
   a.len = st.len;
@@ -467,6 +626,15 @@ cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const v
   a.ring_rows = tc_ring_rows(dm);
   a.qscale = kLog2e / sqrtf((float)dm.d);
   a.skip_copies = g_debug_skip_copies;
+  return a;
+}
+
+cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const void* q, float* out,
+                      int grid, cudaStream_t stream) {
+  const TcMaps* m = static_cast<const TcMaps*>(maps);
+  const TcArgs a = tc_args(st, dm, q, out);
+  FusedArgs f;
+  memset(&f, 0, sizeof(f));
   // programmatic stream serialisation: the grid may be scheduled while the kernel
   // before it (the ingest) finishes; the kernel waits for it before touching the state
   cudaLaunchConfig_t cfg = {};
@@ -481,9 +649,57 @@ cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const v
   if (dm.d == HD_ && dm.G == G_) {                                                        \
     cfg.blockDim = dim3(TcTraits<HD_, G_>::THREADS, 1, 1);                                \
     cfg.dynamicSmemBytes = tc_smem<HD_, G_>(dm.pairs);                                    \
-    return cudaLaunchKernelEx(&cfg, attend_tc_kernel<HD_, G_>, m->sk, m->sv, m->rk, m->rv, a); \
+    return cudaLaunchKernelEx(&cfg, attend_tc_kernel<HD_, G_, false>, m->sk, m->sv, m->rk, \
+                              m->rv, a, f);                                               \
   }
   TC_CASES(LAUNCH)
+#undef LAUNCH
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t tc_launch_fused(const State& st, const Dims& dm, const void* maps, const FusedBufs& fb,
+                            const void* q, const void* k, const void* v, float* out,
+                            const float* override_, int32_t* evict_info, float* score_out, int grid,
+                            cudaStream_t stream) {
+  if (!tc_fused_ok(dm)) return cudaErrorInvalidValue;
+  const TcMaps* m = static_cast<const TcMaps*>(maps);
+  const TcArgs a = tc_args(st, dm, q, out);
+  FusedArgs f;
+  memset(&f, 0, sizeof(f));
+  f.st = st;
+  f.k_new = static_cast<const bf16*>(k);
+  f.v_new = static_cast<const bf16*>(v);
+  f.override_ = override_;
+  f.evict_info = evict_info;
+  f.score_out = score_out;
+  f.part_c = fb.part_c;
+  f.meta_next = fb.meta_next;
+  f.xtra = fb.xtra;
+  f.ctr = fb.ctr;
+  f.batch = dm.batch;
+  f.H = dm.H;
+  f.F = dm.F;
+  f.Fp = dm.Fp;
+  f.s = dm.s;
+  f.act = dm.act;
+  // a programmatic dependent of the step before it: scheduled while that one finishes,
+  // waits for it before reading any state
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+#define LAUNCH(HD_, G_)                                                                    \
+  if (dm.d == HD_ && dm.G == G_) {                                                         \
+    cfg.blockDim = dim3(TcTraits<HD_, G_>::THREADS_F, 1, 1);                               \
+    cfg.dynamicSmemBytes = tc_fused_smem_of(tc_smem<HD_, G_>(dm.pairs), dm.Fp);            \
+    return cudaLaunchKernelEx(&cfg, attend_tc_kernel<HD_, G_, true>, m->sk, m->sv, m->rk,  \
+                              m->rv, a, f);                                                \
+  }
+  TC_FUSED_CASES(LAUNCH)
 #undef LAUNCH
   return cudaErrorInvalidValue;
 }

@@ -20,6 +20,7 @@ enum : int {
   DEVERR_TIMEOUT_DRAIN = 3,    // producer gave up draining its copies at exit
   DEVERR_BAD_SCHEDULE = 4,     // attention schedule inconsistent with the state
   DEVERR_INDEX = 5,            // an index check failed (device-check build only)
+  DEVERR_TIMEOUT_SCHED = 6,    // fused step: gave up waiting for every CTA's schedule
 };
 
 // Index checks of the device-check build (compiled with -DKVPOP_DEVICE_CHECKS):
@@ -164,6 +165,22 @@ cudaError_t tc_make_maps(const State& st, const Dims& dm, void* maps_out);
 cudaError_t tc_config(const Dims& dm, AttendConfig* out);
 cudaError_t tc_launch(const State& st, const Dims& dm, const void* maps, const void* q, float* out,
                       int grid, cudaStream_t stream);
+// The whole decode step in one tensor-core kernel (bf16, d = 128, F <= 256): attention over
+// the keys that cannot change this step while extra warps run the delayed scorer,
+// keep-or-drop and scatter; each pair's last arrival merges.
+struct FusedBufs {
+  float* part_c;               // [pairs][G d + 2 G]
+  int32_t* meta_next;          // [pairs][4]
+  float* xtra;                 // [pairs][2 G + 2 d]
+  int32_t* ctr;                // [2], zero between launches
+};
+bool tc_fused_ok(const Dims& dm);
+int tc_fused_max_grid();         // largest grid the fused kernel's split table holds
+cudaError_t tc_fused_config(const Dims& dm, AttendConfig* out);
+cudaError_t tc_launch_fused(const State& st, const Dims& dm, const void* maps, const FusedBufs& fb,
+                            const void* q, const void* k, const void* v, float* out,
+                            const float* override_, int32_t* evict_info, float* score_out, int grid,
+                            cudaStream_t stream);
 
 // Prefill scores + selection; `tf32_maps` (W1^T tensor maps from prepare_score_tf32, or
 // null) routes the learned scores through the tensor-core scorer.

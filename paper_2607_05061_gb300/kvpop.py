@@ -64,6 +64,7 @@ _SIGS = {
     "kvpop_decode_attend": (ctypes.c_int, [_P, _P, _P, _P]),
     "kvpop_decode_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P]),
     "kvpop_decode_step_host": (ctypes.c_int, [_P, _P, _P, _P, _P, _P]),
+    "kvpop_step_is_fused": (c_int32, [_P]),
     "kvpop_check": (ctypes.c_int, [_P, _P]),
     "kvpop_export_state": (ctypes.c_int, [_P, _P, POINTER(c_size_t), _P]),
     "kvpop_import_state": (ctypes.c_int, [_P, _P, c_size_t, _P]),
@@ -193,6 +194,11 @@ class KVpopCache:
     def step(self, q, k, v, out, override=None, evict_info=None, score_out=None, stream=None):
         _ck(kvpop_decode_step(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(override),
                               _ptr(evict_info), _ptr(score_out), _stream(stream)), "kvpop_decode_step")
+
+    @property
+    def fused_step(self) -> bool:
+        """True when step() runs the whole decode step as one kernel."""
+        return kvpop_step_is_fused(self.handle) == 1
 
     def step_host(self, q, k, v, out, stream=None):
         _ck(kvpop_decode_step_host(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), _stream(stream)),

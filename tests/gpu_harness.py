@@ -15,8 +15,21 @@ TOL = {"f32": 1e-5, "bf16": 2e-2}      # attention max-abs tolerance per K/V dty
 STREAM_PREFILL_OV, STREAM_DECODE_OV = 30, 31
 
 
-def make_cache(cfg, weights, mlstm=None):
+def make_cache(cfg, weights, mlstm=None, step=None):
+    """A cache for `cfg`; step="fused" / "split" forces the one-kernel / two-kernel
+    kvpop_decode_step (default: the library's choice by the size of a step)."""
+    import os
     from paper_2607_05061_gb300 import kvpop
+    if step is not None:
+        saved = {k: os.environ.pop(k, None) for k in ("KVPOP_FUSED_STEP", "KVPOP_SPLIT_STEP")}
+        os.environ["KVPOP_FUSED_STEP" if step == "fused" else "KVPOP_SPLIT_STEP"] = "1"
+        try:
+            return make_cache(cfg, weights, mlstm)
+        finally:
+            for k in ("KVPOP_FUSED_STEP", "KVPOP_SPLIT_STEP"):
+                os.environ.pop(k, None)
+                if saved[k] is not None:
+                    os.environ[k] = saved[k]
     if mlstm is not None:
         return kvpop.KVpopCache(cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim, cfg.budget_B,
                                 cfg.delay_D, cfg.scorer_hidden, cfg.kv_dtype, n_sink=cfg.n_sink,
@@ -64,8 +77,11 @@ class GpuTrace:
 
 
 def gpu_decode(cache, cfg, lengths, nsteps, device, override=None,
-               sample: Optional[Sequence] = None, step0: int = 0) -> GpuTrace:
-    """Run ``nsteps`` decode steps; keep outputs of the sampled (b, h) pairs (all if None)."""
+               sample: Optional[Sequence] = None, step0: int = 0, split: bool = False) -> GpuTrace:
+    """Run ``nsteps`` decode steps; keep outputs of the sampled (b, h) pairs (all if None).
+
+    Each step is one kvpop_decode_step call (one kernel where the cache supports it), or
+    with ``split`` a kvpop_decode_ingest and a kvpop_decode_attend call."""
     b, H, G, d = cfg.batch, cfg.n_kv_heads, cfg.q_per_kv, cfg.head_dim
     q, k, v = gen.decode_inputs(cfg, lengths, step0, nsteps, device=device)
     out = torch.empty((b, H * G, d), dtype=torch.float32, device=device)
@@ -76,8 +92,11 @@ def gpu_decode(cache, cfg, lengths, nsteps, device, override=None,
     outs = torch.empty((nsteps, len(pairs), G, d), dtype=torch.float32, device=device)
     for j in range(nsteps):
         ov = None if override is None else override[j]
-        cache.ingest(q[j], k[j], v[j], override=ov, evict_info=ei[j], score_out=sc[j])
-        cache.attend(q[j], out)
+        if split:
+            cache.ingest(q[j], k[j], v[j], override=ov, evict_info=ei[j], score_out=sc[j])
+            cache.attend(q[j], out)
+        else:
+            cache.step(q[j], k[j], v[j], out, override=ov, evict_info=ei[j], score_out=sc[j])
         outs[j] = out.view(b * H, G, d).index_select(0, sel)
     torch.cuda.synchronize()
     cache.check()

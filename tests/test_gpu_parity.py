@@ -102,7 +102,10 @@ SMALL = dict(batch=2, prompt_len=600, budget_B=256, decode_steps=200)
                   decode_steps=120)),
     ("tiny", dict(q_per_kv=1, prompt_len=90, budget_B=16, delay_D=2, decode_steps=90)),
 ])
-def test_injected_scores_bitexact(cuda_device, name, over):
+@pytest.mark.parametrize("path", ["fused", "split"])
+def test_injected_scores_bitexact(cuda_device, name, over, path):
+    """Every case on both kvpop_decode_step paths (one kernel where the shape allows it:
+    bf16, d = 128; the fp32 and d = 64 cases run the two-kernel path either way)."""
     cfg = get_config(name, **over)
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
@@ -111,14 +114,114 @@ def test_injected_scores_bitexact(cuda_device, name, over):
     Pmax = max(1, max(L))
     pov = injected_prefill_scores(cfg, Pmax, "cpu")
     dov = injected_decode_scores(cfg, steps, "cpu")
-    cache = make_cache(cfg, w)
+    cache = make_cache(cfg, w, step=path)
     gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
     g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device))
     ref = oracle_pairs(cfg, w, L, steps, pairs, prefill_override=pov, decode_override=dov)
     err = compare(cfg, g, ref, pairs)
-    print(f"{name} {over}: max-abs attention error {err:.3e}")
+    print(f"{name} {over} {path} (one kernel: {cache.fused_step}): max-abs attention error {err:.3e}")
     assert err <= TOL[cfg.kv_dtype]
     cache.free()
+
+
+def test_fused_step_selected(cuda_device):
+    """kvpop_decode_step is one kernel for bf16, d = 128, F = 256 when a step streams at
+    least 600 MB of K/V (cr8x: 1.08 GB) or when asked; two kernels for a small stream
+    (q4b: 0.10 GB), d = 64, fp32, or when asked."""
+    def fused(name, step=None, **over):
+        cfg = get_config(name, **over)
+        c = make_cache(cfg, gen.scorer_weights(cfg), step=step)
+        f = c.fused_step
+        c.free()
+        return f
+    assert fused("cr8x", prompt_len=64)
+    assert not fused("q4b")
+    assert fused("q4b", step="fused", **SMALL)
+    assert not fused("q4b", step="fused", **dict(SMALL, q_per_kv=1, head_dim=64))
+    assert not fused("tiny", step="fused")
+    assert not fused("cr8x", step="split", prompt_len=64)
+
+
+@pytest.mark.parametrize("name,over", [
+    ("q4b", SMALL),
+    ("q4b", dict(SMALL, prompt_len=5, decode_steps=80, n_sink=2)),
+])
+def test_split_step_bitexact(cuda_device, name, over):
+    """The two-call path (kvpop_decode_ingest + kvpop_decode_attend) on a cache whose
+    kvpop_decode_step is one kernel: the same oracle bar."""
+    cfg = get_config(name, **over)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    steps = cfg.decode_steps
+    pov = injected_prefill_scores(cfg, max(1, max(L)), "cpu")
+    dov = injected_decode_scores(cfg, steps, "cpu")
+    cache = make_cache(cfg, w, step="fused")
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device), split=True)
+    ref = oracle_pairs(cfg, w, L, steps, pairs, prefill_override=pov, decode_override=dov)
+    assert compare(cfg, g, ref, pairs) <= TOL[cfg.kv_dtype]
+    cache.free()
+
+
+def test_fused_partial_scorer_group(cuda_device):
+    """20 sequences: two scorer units per KV head, the second with 4 of 16 rows."""
+    cfg = get_config("q4b", batch=20, prompt_len=400, budget_B=128, decode_steps=64)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    pairs = all_pairs(cfg)
+    steps = cfg.decode_steps
+    pov = injected_prefill_scores(cfg, max(L), "cpu")
+    dov = injected_decode_scores(cfg, steps, "cpu")
+    cache = make_cache(cfg, w, step="fused")
+    assert cache.fused_step
+    gpu_prefill(cache, cfg, L, cuda_device, override=pov.to(cuda_device))
+    g = gpu_decode(cache, cfg, L, steps, cuda_device, override=dov.to(cuda_device))
+    ref = oracle_pairs(cfg, w, L, steps, pairs, prefill_override=pov, decode_override=dov)
+    err = compare(cfg, g, ref, pairs)
+    print(f"q4b b20: max-abs attention error {err:.3e}")
+    assert err <= TOL["bf16"]
+    cache.free()
+
+
+def test_fused_and_split_own_scores(cuda_device):
+    """Each path scoring on its own: the fused scorer against the oracle's scores (rel
+    2e-5, the fp32-accurate bound of every scorer check), and both paths' outputs within
+    the bf16 tolerance of each other."""
+    cfg = get_config("q4b", batch=18, prompt_len=700, budget_B=256, decode_steps=48)
+    w = gen.scorer_weights(cfg)
+    L = gen.prompt_lengths(cfg)
+    steps = cfg.decode_steps
+    a = make_cache(cfg, w, step="fused")
+    b = make_cache(cfg, w, step="split")
+    assert a.fused_step and not b.fused_step
+    gpu_prefill(a, cfg, L, cuda_device)
+    gpu_prefill(b, cfg, L, cuda_device)
+    ga = gpu_decode(a, cfg, L, steps, cuda_device)
+    gb = gpu_decode(b, cfg, L, steps, cuda_device)
+    sample = [(0, 0), (17, 7)]
+    ref = oracle_pairs(cfg, w, L, steps, sample, attend=False)
+    for (bb, hh), tr in zip(sample, ref):
+        want = np.asarray(tr.scores, dtype=np.float64)
+        got = ga.scores[:, bb, hh].astype(np.float64)
+        rel = np.abs(got - want) / (1.0 + np.abs(want))
+        assert np.all(rel <= 2e-5), f"fused scorer {(bb, hh)}: {np.nanmax(rel):.2e}"
+    eq = (ga.evict == gb.evict).all(axis=-1)              # [steps][b][H]
+    same = eq.mean()
+    # outputs compared up to a pair's first differing decision (a near-tie decided the
+    # other way by the last bit of a score changes the kept set from then on)
+    diff = 0.0
+    for bb in range(cfg.batch):
+        for hh in range(cfg.n_kv_heads):
+            bad = np.nonzero(~eq[:, bb, hh])[0]
+            n = int(bad[0]) if bad.size else steps
+            if n:
+                i = bb * cfg.n_kv_heads + hh
+                diff = max(diff, float(np.abs(ga.outputs[:n, i] - gb.outputs[:n, i]).max()))
+    print(f"fused vs split, own scores: decisions equal {same:.4f}, max-abs output difference {diff:.2e}")
+    assert diff <= TOL["bf16"]
+    a.free()
+    b.free()
 
 
 def test_planted_ties_bitexact(cuda_device):
@@ -171,14 +274,16 @@ def test_full_size_sampled(cuda_device, name, steps, sample):
     cache.free()
 
 
-def test_full_size_gpu_scorer(cuda_device):
-    """cr8x shape, GPU scorer: per-token scores vs the oracle scorer on sampled pairs."""
+@pytest.mark.parametrize("path", ["fused", "split"])
+def test_full_size_gpu_scorer(cuda_device, path):
+    """cr8x shape, GPU scorer (of either kvpop_decode_step path): per-token scores vs the
+    oracle scorer on sampled pairs."""
     cfg = get_config("cr8x", batch=8)
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
     steps = 32
     sample = [(0, 0), (5, 3)]
-    cache = make_cache(cfg, w)
+    cache = make_cache(cfg, w, step=path)
     gpu_prefill(cache, cfg, L, cuda_device)
     g = gpu_decode(cache, cfg, L, steps, cuda_device, sample=sample)
     ref = oracle_pairs(cfg, w, L, steps, sample, attend=False)

@@ -32,7 +32,9 @@ def prefill_stack(st, cfg, L, device, overrides=None):
         st.prefill_layer(l, X, L, override=ov)
 
 
-def test_stack_matches_oracle_stack(cuda_device):
+@pytest.mark.parametrize("path", ["fused", "split"])
+def test_stack_matches_oracle_stack(cuda_device, monkeypatch, path):
+    """Both kvpop_decode_step paths (the full-size stack runs the one-kernel step)."""
     from oracle.stack import run_stack
     cfg = get_config("q8b_stack", **SMALL_STACK)
     L = gen.prompt_lengths(cfg)
@@ -40,7 +42,13 @@ def test_stack_matches_oracle_stack(cuda_device):
     b, H, Hq, d = cfg.batch, cfg.n_kv_heads, cfg.n_q_heads, cfg.head_dim
     pov = [gen.uniform_scores(cfg.seed, 70 + l, (b, H, max(L))) for l in range(cfg.n_layers)]
     dov = [gen.uniform_scores(cfg.seed, 80 + l, (steps, b, H)) for l in range(cfg.n_layers)]
+    monkeypatch.delenv("KVPOP_FUSED_STEP", raising=False)
+    monkeypatch.delenv("KVPOP_SPLIT_STEP", raising=False)
+    monkeypatch.setenv("KVPOP_FUSED_STEP" if path == "fused" else "KVPOP_SPLIT_STEP", "1")
     st = build_stack(cfg, cuda_device)
+    monkeypatch.delenv("KVPOP_FUSED_STEP", raising=False)
+    monkeypatch.delenv("KVPOP_SPLIT_STEP", raising=False)
+    assert all(c.fused_step == (path == "fused") for c in st.caches)
     prefill_stack(st, cfg, L, cuda_device, pov)
     xs = gen.decode_hidden(cfg, L, 0, steps, device=cuda_device)
     outs = [torch.empty((b, Hq * d), device=cuda_device) for _ in range(cfg.n_layers)]
