@@ -288,16 +288,17 @@ constexpr int T6_HALF = 128;
 constexpr int T6_ROWS = 2 * T6_HALF;            // keys per CTA
 constexpr int T6_BN = 128;                      // queries per block (MMA N)
 constexpr int T6_ST = 4;                        // query-block stages
-constexpr int T6_MMA_WARP = 8;                  // warps 0-7 softmax, 8 MMA, 9-11 producers
+constexpr int T6_MMA_WARP = 16;                 // warps 0-15 softmax, 16 MMA, 17-19 producers
 constexpr int T6_PT = 96;
-constexpr int T6_THREADS = 32 * 12;
+constexpr int T6_THREADS = 32 * 20;
 constexpr int T6_KB = T6_HALF * 256;            // key tile of one half
 constexpr int T6_QB = T6_BN * 256;              // query block
 constexpr int T6_OFF_Q = 2 * T6_KB;
 constexpr int T6_OFF_LSE = T6_OFF_Q + T6_ST * T6_QB;
 constexpr int T6_OFF_BAR = T6_OFF_LSE + T6_ST * T6_BN * 4;
 constexpr int T6_OFF_TMEM = T6_OFF_BAR + 8 * 32;
-constexpr int T6_SMEM = T6_OFF_TMEM + 16;
+constexpr int T6_OFF_PX = T6_OFF_TMEM + 16;      // [2 head parity][2 halves][128 rows][m, l, seq, -]
+constexpr int T6_SMEM = T6_OFF_PX + 2 * 2 * T6_HALF * 16;
 constexpr int T6_FULL = 0, T6_EMPTY = T6_ST, T6_SFULL = 2 * T6_ST, T6_PFULL = 2 * T6_ST + 4,
               T6_KFULL = 2 * T6_ST + 8;
 enum : int { T6ERR_WAIT = 22 };
@@ -329,14 +330,17 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
   if (tid == 0) {
     for (int i = 0; i < T6_ST; ++i) {
       mbar_init(bar(T6_FULL + i), 2 * T6_PT);            // cp.async arrivals + plain stores
-      mbar_init(bar(T6_EMPTY + i), 1 + 2 * T6_HALF);   // MMA commit + every softmax thread (LSE)
+      mbar_init(bar(T6_EMPTY + i), 1 + 4 * T6_HALF);   // MMA commit + every softmax thread (LSE)
     }
     for (int i = 0; i < 4; ++i) {
       mbar_init(bar(T6_SFULL + i), 1);
-      mbar_init(bar(T6_PFULL + i), T6_HALF);
+      mbar_init(bar(T6_PFULL + i), 2 * T6_HALF);
     }
     mbar_init(bar(T6_KFULL), T6_PT);
     mbar_fence_init();
+    // the softmax halves' exchange slots start with no head done
+    int* px = reinterpret_cast<int*>(sm6 + T6_OFF_PX);
+    for (int i = 0; i < 2 * 2 * T6_HALF; ++i) px[4 * i + 2] = 0;
   }
   if (warp == T6_MMA_WARP) tmem_alloc(sb + T6_OFF_TMEM, 512);
   fence_before();
@@ -407,12 +411,18 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
     __syncwarp();
   } else {
     // ---------------------------------------------------------------- softmax rows
-    const int hh = warp >> 2;
+    // warp w: half hh = (w / 4) mod 2 of the CTA's keys, key row r = 32 (w mod 4) + lane (the
+    // warp's tensor-memory lane quarter), and columns [64 cs, 64 cs + 64) of every block with
+    // cs = w / 8: four warps per subpartition share the exponentials of a block.  The two
+    // column halves of a row keep their own (max, sum) over a head's blocks and meet at the
+    // head's end in shared memory.
+    const int hh = (warp >> 2) & 1, cs = warp >> 3;
     const int r = (warp & 3) * 32 + lane;
     const int t = t0 + hh * T6_HALF + r;
     const int hi = t <= t1 ? future_hi(t, L, w, la) : -1;
     const uint32_t tS = tmem + ((uint32_t)((warp & 3) * 32) << 16) + hh * 256;
     const float* nlS = reinterpret_cast<const float*>(sm6 + T6_OFF_LSE);   // -log2(e) LSE_d per stage
+    float* pxs = reinterpret_cast<float*>(sm6 + T6_OFF_PX);
     const float c2 = a.kscale;
     float m = -INFINITY, l = 0.f;
     auto uniform = [](bool x) { return __all_sync(0xffffffffu, x); };
@@ -424,23 +434,23 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
       // the stage's normalisers (complete long before S; the wait orders their reads)
       if (!uniform(mbar_wait(bar(T6_FULL + st), (j / T6_ST) & 1, a.err, T6ERR_WAIT))) break;
       fence_after();
-      // the block's 128 columns as two 64-column halves, each folded into the running sum
+      // this thread's 64 columns as two 32-column parts, each folded into the running sum
 #pragma unroll 1
       for (int c = 0; c < 2; ++c) {
-        const int e0 = d0 + 64 * c;
-        float s[64];
-        tmem_ld32(tS + b2 * T6_BN + 64 * c, *reinterpret_cast<float(*)[32]>(s));
-        tmem_ld32(tS + b2 * T6_BN + 64 * c + 32, *reinterpret_cast<float(*)[32]>(s + 32));
+        const int col = 64 * cs + 32 * c;
+        const int e0 = d0 + col;
+        float s[32];
+        tmem_ld32(tS + b2 * T6_BN + col, s);
         tmem_wait_ld();
         if (c == 1) {
-          // the S buffer is in registers: the MMA may overwrite it
+          // the thread's part of the S buffer is in registers: the MMA may overwrite it
           fence_before();
           mbar_arrive(bar(T6_PFULL + 2 * hh + b2));
         }
-        const bool masked = e0 < t1 + w || e0 + 63 > d_hi || (la > 0 && e0 + 63 > t0 + w + la);
+        const bool masked = e0 < t1 + w || e0 + 31 > d_hi || (la > 0 && e0 + 31 > t0 + w + la);
         if (masked) {                               // on the raw logits: -inf c2 + n = -inf
 #pragma unroll
-          for (int i = 0; i < 64; ++i) {
+          for (int i = 0; i < 32; ++i) {
             const int d = e0 + i;
             if (d < t + w || d > hi) s[i] = -INFINITY;
           }
@@ -448,15 +458,13 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         // x = s c2 - log2(e) LSE_d is the query's log2 attention probability of the key, so
         // 2^x needs no running maximum unless the key lies outside the query's kept set
         // with a much larger logit: sum with base 0, and take the maximum only when the
-        // half's sum leaves [2^-60, 2^60] (overflow, NaN, or every term tiny or masked).
-        // One loop forms x (packed FMA, kept in s for that case) and feeds the exponentials,
-        // so the FMA work issues under the MUFU's.
+        // part's sum leaves [2^-60, 2^60] (overflow, NaN, or every term tiny or masked).
         {
-          const float4* l4 = reinterpret_cast<const float4*>(nlS + st * T6_BN + 64 * c);
+          const float4* l4 = reinterpret_cast<const float4*>(nlS + st * T6_BN + col);
           const uint64_t cc = f2_pack(c2, c2);
           uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-          for (int i4 = 0; i4 < 16; ++i4) {
+          for (int i4 = 0; i4 < 8; ++i4) {
             const float4 v = l4[i4];
             f2_unpack(f2_fma(f2_pack(s[4 * i4], s[4 * i4 + 1]), cc, f2_pack(v.x, v.y)), s[4 * i4],
                       s[4 * i4 + 1]);
@@ -466,7 +474,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
             ps[k] = f2_add(ps[k], f2_pack(ex2(s[4 * i4]), ex2(s[4 * i4 + 1])));
             ps[k + 1] = f2_add(ps[k + 1], f2_pack(ex2(s[4 * i4 + 2]), ex2(s[4 * i4 + 3])));
           }
-          // the stage's query rows and normalisers are no longer needed
+          // the stage's query rows and normalisers are no longer needed by this thread
           if (c == 1) mbar_arrive(bar(T6_EMPTY + st));
           float q[8];
 #pragma unroll
@@ -482,14 +490,14 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
             continue;
           }
         }
-        // row maximum: 8 chains of three-input maxima
+        // part maximum: 8 chains of three-input maxima
         float pm[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) pm[k] = s[k];
 #pragma unroll
-        for (int i = 8; i < 64; i += 16)
+        for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[8 + k], s[16 + k]);
 #pragma unroll
-          for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+        for (int k = 0; k < 8; ++k) pm[k] = fmaxf(pm[k], s[24 + k]);
         const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
         const float mn = fmaxf(m, mx);
         const float base = mn == -INFINITY ? 0.f : mn;
@@ -497,7 +505,7 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         const uint64_t nb = f2_pack(-base, -base);
         uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-        for (int i = 0; i < 64; i += 8) {
+        for (int i = 0; i < 32; i += 8) {
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             float x0, x1;
@@ -511,8 +519,31 @@ __global__ void __launch_bounds__(T6_THREADS, 1) target_t5_kernel(TargetArgs a) 
         l = l * ex2(m - base) + (((q[0] + q[1]) + (q[2] + q[3])) + ((q[4] + q[5]) + (q[6] + q[7])));
         m = mn;
       }
-      if (b == nblk - 1) {                          // head g done: write and reset
-        if (t <= t1) a.logm[(qrow0 + g) * S + t] = l > 0.f ? (m + __log2f(l)) * kLn2f : -INFINITY;
+      if (b == nblk - 1) {
+        // head g done: the upper column half hands its (max, sum) to the lower, which merges
+        // and writes the key's log mass (slots alternate by head; a flag names the head)
+        float* px = pxs + (((size_t)(g & 1) * 2 + hh) * T6_HALF + r) * 4;
+        volatile int* seq = reinterpret_cast<volatile int*>(px) + 2;
+        if (cs == 1) {
+          px[0] = m;
+          px[1] = l;
+          __threadfence_block();
+          *seq = g + 1;
+        } else {
+          bool ready = *seq == g + 1;
+          if (!ready) {
+            const unsigned long long tw = globaltimer();
+            while (!(ready = *seq == g + 1))
+              if (globaltimer() - tw > kWaitLimitNs) { atomicCAS(a.err, 0, T6ERR_WAIT); break; }
+          }
+          __threadfence_block();
+          const float m1 = px[0], l1 = px[1];
+          const float M = fmaxf(m, m1);
+          float Lr = 0.f;
+          if (M != -INFINITY)
+            Lr = (m == -INFINITY ? 0.f : l * ex2(m - M)) + (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - M));
+          if (t <= t1) a.logm[(qrow0 + g) * S + t] = Lr > 0.f ? (M + __log2f(Lr)) * kLn2f : -INFINITY;
+        }
         m = -INFINITY;
         l = 0.f;
       }
