@@ -117,7 +117,8 @@ __device__ bool tile_setup(const PromptArgs& a, int BM, int* tauS, int* red, int
         ca += r[e] <= tmin;
         cm += (r[e] > tmin) & (r[e] <= tmax);
       }
-      const int v = ca | (cm << 16);        // at most NT * EPT = 6144 per field
+      static_assert(NT * EPT < 65536, "two 16-bit counts per word");
+      const int v = ca | (cm << 16);        // at most NT * EPT per field
       int x = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {

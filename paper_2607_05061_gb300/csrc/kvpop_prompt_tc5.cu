@@ -43,6 +43,7 @@ constexpr int T5_MMA_WARP = 8;                   // warps 0-7: softmax, 8: MMA, 
 constexpr int T5_NPROD = 3;
 constexpr int T5_PT = 32 * T5_NPROD;
 constexpr int T5_THREADS = 32 * (T5_MMA_WARP + 1 + T5_NPROD);   // 12 warps: 168 registers fit
+static_assert(T5_THREADS / 32 + 2 <= 16, "the prologue's per-warp reduction slots");
 constexpr int T5_TMEM_COLS = 512;                // O_h: 128 h .. ; S_{h,b}: 256 + 128 h + 64 b
 constexpr float T5_THR = 8.0f;
 
@@ -240,9 +241,11 @@ __global__ void __launch_bounds__(T5_THREADS, 1) prompt_t5_kernel(PromptArgs a) 
 #pragma unroll
         for (int k = 0; k < 8; ++k) pm[k] = s[k];
 #pragma unroll
-        for (int i = 8; i < 64; i += 16)
+        for (int i = 8; i < 56; i += 16)
 #pragma unroll
           for (int k = 0; k < 8; ++k) pm[k] = fmax3(pm[k], s[i + k], s[i + 8 + k]);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) pm[k] = fmaxf(pm[k], s[56 + k]);
         const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
         const float mxs = mx * c2;                  // row maximum, log2 units
         float alpha = 1.f, m_new = m;
