@@ -552,8 +552,8 @@ def run_kvpop(args):
                      "ms_per_launch_how": attn_how},
         "e2e": {"value": tokens_per_step / (e2e_max / 1e3), "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": E,
-                "how": "kvpop_decode_step_host on pinned host buffers (q|k|v packed: one copy in; "
-                       "the attention writes out into pinned host memory), stream sync every step"
+                "how": "kvpop_decode_step_host on pinned host buffers: the step's kernels read q|k|v "
+                       "and write out in place over NVLink-C2C; stream sync every step"
                        + ("; L2 flushed before each step, outside its timing" if flush else "")},
         "gpu_launches": K if fused else 2 * K,
         "clocks": clk,

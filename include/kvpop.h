@@ -318,11 +318,13 @@ kvpop_status kvpop_decode_step(kvpop_cache* cache, const void* q_dev, const void
  * ingest and the attention as two, -1 for an invalid handle. */
 int32_t kvpop_step_is_fused(const kvpop_cache* cache);
 
-/* kvpop_decode_step on host buffers (pinned memory recommended): copies q/k/v
- * into library-owned device staging (one copy when k_host and v_host follow q_host
- * directly in one buffer), runs the step and returns out, all on `stream` (the
- * caller synchronises before reading out_host).  When out_host is pinned memory the
- * device can address, the attention writes it directly; otherwise it is copied
+/* kvpop_decode_step on host buffers (pinned memory recommended), all on `stream`
+ * (the caller synchronises before reading out_host or reusing the inputs).  When
+ * q_host, k_host and v_host are all pinned memory the device can address (on
+ * Grace-Blackwell over NVLink-C2C), the step's kernels read them in place;
+ * otherwise they are copied into library-owned device staging first (one copy when
+ * k_host and v_host follow q_host directly in one buffer).  Likewise the attention
+ * writes a device-addressable pinned out_host directly, and anything else is copied
  * back from device staging. */
 kvpop_status kvpop_decode_step_host(kvpop_cache* cache, const void* q_host, const void* k_host,
                                     const void* v_host, float* out_host, cudaStream_t stream);

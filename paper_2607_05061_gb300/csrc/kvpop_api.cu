@@ -91,6 +91,18 @@ kvpop_status from_cuda(cudaError_t e) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
+// Device address of pinned host memory the device can address in place (NVLink-C2C /
+// PCIe mapping) and 16-byte aligned there; NULL for anything else.
+const void* mapped_host(const void* p) {
+  cudaPointerAttributes pa{};
+  const void* d = nullptr;
+  if (cudaPointerGetAttributes(&pa, p) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+      pa.devicePointer != nullptr && aligned16(pa.devicePointer))
+    d = pa.devicePointer;
+  cudaGetLastError();   // a pointer the runtime does not know is not an error here
+  return d;
+}
+
 kvpop_status dev_alloc(kvpop_cache* c, void** p, size_t bytes) {
   *p = nullptr;
   if (g_fail_after > 0 && --g_fail_after == 0) return KVPOP_ERR_OOM;
@@ -768,32 +780,35 @@ kvpop_status kvpop_decode_step_host(kvpop_cache* c, const void* q, const void* k
   if (!q || !k || !v || !out) return KVPOP_ERR_INVALID_ARG;
   const size_t pairs = c->dm.pairs, d = c->dm.d, G = c->dm.G;
   const size_t qb = pairs * G * d * c->esz, kb = pairs * d * c->esz;
-  const char* qc = static_cast<const char*>(q);
-  cudaError_t e = cudaErrorInvalidValue;
-  // adjacent buffers take one copy; adjacent addresses from different host allocations
-  // are refused by the runtime before anything is queued, and then take three
-  if (static_cast<const char*>(k) == qc + qb && static_cast<const char*>(v) == qc + qb + kb) {
-    e = cudaMemcpyAsync(c->stage_q, q, qb + 2 * kb, cudaMemcpyHostToDevice, stream);
-    if (e == cudaErrorInvalidValue) cudaGetLastError();
+  // pinned host memory the device can address is read (inputs) and written (output) by
+  // the step's kernels in place; anything else goes through the device staging buffers
+  const void* mq = mapped_host(q);
+  const void* mk = mq ? mapped_host(k) : nullptr;
+  const void* mv = mk ? mapped_host(v) : nullptr;
+  float* direct = static_cast<float*>(const_cast<void*>(mapped_host(out)));
+  const void *dq = mq, *dk = mk, *dv = mv;
+  if (!mv) {
+    const char* qc = static_cast<const char*>(q);
+    cudaError_t e = cudaErrorInvalidValue;
+    // adjacent buffers take one copy; adjacent addresses from different host allocations
+    // are refused by the runtime before anything is queued, and then take three
+    if (static_cast<const char*>(k) == qc + qb && static_cast<const char*>(v) == qc + qb + kb) {
+      e = cudaMemcpyAsync(c->stage_q, q, qb + 2 * kb, cudaMemcpyHostToDevice, stream);
+      if (e == cudaErrorInvalidValue) cudaGetLastError();
+    }
+    if (e == cudaErrorInvalidValue) {
+      e = NOTE(cudaMemcpyAsync(c->stage_q, q, qb, cudaMemcpyHostToDevice, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_k, k, kb, cudaMemcpyHostToDevice, stream));
+      if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_v, v, kb, cudaMemcpyHostToDevice, stream));
+    }
+    if (e != cudaSuccess) return poison_on(c, e);
+    dq = c->stage_q;
+    dk = c->stage_k;
+    dv = c->stage_v;
   }
-  if (e == cudaErrorInvalidValue) {
-    e = NOTE(cudaMemcpyAsync(c->stage_q, q, qb, cudaMemcpyHostToDevice, stream));
-    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_k, k, kb, cudaMemcpyHostToDevice, stream));
-    if (e == cudaSuccess) e = NOTE(cudaMemcpyAsync(c->stage_v, v, kb, cudaMemcpyHostToDevice, stream));
-  }
-  if (e != cudaSuccess) return poison_on(c, e);
-  // pinned host memory the device can address (NVLink-C2C / PCIe mapping) takes the
-  // attention output directly; anything else goes through the device staging buffer
-  cudaPointerAttributes pa{};
-  float* direct = nullptr;
-  if (cudaPointerGetAttributes(&pa, out) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
-      pa.devicePointer != nullptr && aligned16(pa.devicePointer))
-    direct = static_cast<float*>(pa.devicePointer);
-  cudaGetLastError();   // a pointer the runtime does not know is not an error here
-  s = kvpop_decode_step(c, c->stage_q, c->stage_k, c->stage_v, direct ? direct : c->stage_out,
-                        nullptr, nullptr, nullptr, stream);
+  s = kvpop_decode_step(c, dq, dk, dv, direct ? direct : c->stage_out, nullptr, nullptr, nullptr, stream);
   if (s != KVPOP_OK || direct) return s;
-  e = NOTE(cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream));
+  cudaError_t e = NOTE(cudaMemcpyAsync(out, c->stage_out, pairs * G * d * 4, cudaMemcpyDeviceToHost, stream));
   return poison_on(c, e);
 }
 

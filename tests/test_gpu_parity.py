@@ -324,15 +324,21 @@ def test_checkpoint_resume_is_bit_identical(cuda_device):
     b.free()
 
 
-@pytest.mark.parametrize("packed,pinned_out", [(False, True), (True, False), (True, True)])
-def test_host_buffer_step_matches_device_step(cuda_device, packed, pinned_out):
-    """kvpop_decode_step_host equals the device step bit for bit: separate or packed
-    (q | k | v in one buffer, one copy) inputs; output written by the attention into
-    pinned host memory or copied back from device staging (pageable output)."""
+@pytest.mark.parametrize("inputs,pinned_out,step", [
+    ("pinned", True, None), ("packed", False, None), ("packed", True, None),
+    ("pageable", True, None), ("packed_pageable", False, None),
+    ("packed", True, "fused"), ("pageable", False, "fused")])
+def test_host_buffer_step_matches_device_step(cuda_device, inputs, pinned_out, step):
+    """kvpop_decode_step_host equals the device step bit for bit, on the two-kernel and
+    the one-kernel path: pinned inputs (separate, or q | k | v in one buffer) read in
+    place by the kernels, pageable inputs copied in (three copies, or one when packed);
+    output written by the attention into pinned host memory or copied back from device
+    staging (pageable output)."""
     cfg = get_config("q4b", batch=2, prompt_len=300, budget_B=64, decode_steps=20)
     w = gen.scorer_weights(cfg)
     L = gen.prompt_lengths(cfg)
-    a, b = make_cache(cfg, w), make_cache(cfg, w)
+    a, b = make_cache(cfg, w, step=step), make_cache(cfg, w, step=step)
+    assert a.fused_step == (step == "fused")
     gpu_prefill(a, cfg, L, cuda_device)
     gpu_prefill(b, cfg, L, cuda_device)
     q, k, v = gen.decode_inputs(cfg, L, 0, 20, device="cpu")
@@ -340,17 +346,20 @@ def test_host_buffer_step_matches_device_step(cuda_device, packed, pinned_out):
     out_h = torch.empty((cfg.batch, cfg.n_q_heads, cfg.head_dim))
     out_h = out_h.pin_memory() if pinned_out else out_h
     qb, kb = q[0].numel() * q.element_size(), k[0].numel() * k.element_size()
-    buf = torch.empty(qb + 2 * kb, dtype=torch.uint8).pin_memory()
+    buf = torch.empty(qb + 2 * kb, dtype=torch.uint8)
+    buf = buf if inputs == "packed_pageable" else buf.pin_memory()
     for j in range(20):
         a.step(q[j].to(cuda_device), k[j].to(cuda_device), v[j].to(cuda_device), out_d)
-        if packed:
+        if inputs.startswith("packed"):
             hq = buf[:qb].view(q.dtype).view(q[j].shape)
             hk = buf[qb:qb + kb].view(k.dtype).view(k[j].shape)
             hv = buf[qb + kb:].view(v.dtype).view(v[j].shape)
             hq.copy_(q[j]); hk.copy_(k[j]); hv.copy_(v[j])
             b.step_host(hq, hk, hv, out_h)
-        else:
+        elif inputs == "pinned":
             b.step_host(q[j].pin_memory(), k[j].pin_memory(), v[j].pin_memory(), out_h)
+        else:
+            b.step_host(q[j].clone(), k[j].clone(), v[j].clone(), out_h)
         torch.cuda.synchronize()
         assert torch.equal(out_d.cpu(), out_h)
     a.free()
