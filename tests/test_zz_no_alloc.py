@@ -29,7 +29,7 @@ def caller_buffers(cache, device):
     """Device copies, owned by the caller, of the cache state the entry point reads."""
     from paper_2607_05061_gb300 import kvpop
     st = kvpop.parse_state(cache.export_state(), cache.cfg)
-    return {k: torch.from_numpy(np.ascontiguousarray(st[k])).to(device) for k in STATE_FIELDS}
+    return {k: torch.from_numpy(np.array(st[k], copy=True)).to(device) for k in STATE_FIELDS}
 
 
 def sampled_pairs(cfg, n=4):
