@@ -196,6 +196,7 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
   // the CTAs with one scorer unit more than the rest stream 3/64 fewer tiles (when every
   // CTA has at least 4)
   int* bnd = reinterpret_cast<int*>(smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::BND);
+  int* sched_seen = reinterpret_cast<int*>(smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::FLAG);
   Split sp{Ttot, NC, bnd};
   if constexpr (FUSED) {
     const int units = f.H * ((f.batch + kFusedSeqs - 1) / kFusedSeqs);
@@ -203,6 +204,7 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
     const bool weigh = Ttot >= 4 * NC && extra > 0;
     split_bounds(bnd, Ttot, NC, weigh ? (int)min((long long)extra, NC) : 0, weigh ? KVPOP_FUSED_SPLIT_K : 0,
                  tid, NT);
+    if (tid == 0) *sched_seen = 0;
     __syncthreads();
   }
   const bool streams = Ttot > 0 && blockIdx.x < NC;
@@ -387,7 +389,7 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
       if (last) {
         __threadfence();
         fused_merge<HD, G, NCT>(f, a.out, a.part, a.part_count, p, prefix, sp, (long long)blockIdx.x,
-                                om, ol, oo, tid, [] { consumer_sync(); });
+                                om, ol, oo, tid, sched_seen, [] { consumer_sync(); });
       }
       consumer_sync();
     }

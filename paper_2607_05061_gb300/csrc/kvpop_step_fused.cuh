@@ -53,7 +53,7 @@ struct FusedSmem {
   static constexpr int SEQ = RP + kFusedSW * kFusedSeqs * 4;   // [4][16] len, nvalid, min, min slot
   static constexpr int SXC = SEQ + 4 * kFusedSeqs * 4;   // [4][2] extra-key logits (consumers)
   static constexpr int SXS = SXC + 32;                   // (spare)
-  static constexpr int FLAG = SXS + kFusedSW * 32;       // int flags
+  static constexpr int FLAG = SXS + kFusedSW * 32;       // int flags: [0] every CTA's schedule built
   static constexpr int BND = FLAG + 16;                  // [kMaxSplit + 1] ints: CTA ranges
   static constexpr int WBAR = BND + (kMaxSplit + 1) * 4 + 4;   // [3] mbarriers of the weight ring
   static constexpr int W1R = (WBAR + 24 + 127) & ~127;   // [3][kW1Rows][Fp] weight ring
@@ -68,6 +68,16 @@ __host__ __device__ inline size_t fused_smem_bytes(int Fp) {
 __device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// CTA-scope release / acquire on a shared-memory flag (a fact one warp established
+// passed on to the others of the CTA, with its ordering)
+__device__ __forceinline__ void st_release_cta(int* p, int v) {
+  asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_cta(const int* p) {
+  int v;
+  asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
   return v;
 }
 
@@ -164,10 +174,14 @@ struct MergeShape {
 template <int HD, int G, int NTHR, typename SyncFn>
 __device__ void fused_merge(const FusedArgs& f, float* out, const float* part, int32_t* part_count,
                             int p, const int* prefix, const Split& sp, long long own_cta, const float* own_m, const float* own_l,
-                            const float* own_o, int tid, SyncFn sync) {
+                            const float* own_o, int tid, int* sched_seen, SyncFn sync) {
   constexpr int EPT = MergeShape<HD, G, NTHR>::EPT;
   constexpr int NE = G * HD;
   const State& st = f.st;
+  // the pair's next length, used slots and minimum: written by the scorer before its
+  // arrival, which the caller has acquired, so loaded now beside the partials
+  int4 mt = make_int4(0, 0, 0, 0);
+  if (tid == 0) mt = __ldcg(reinterpret_cast<const int4*>(f.meta_next) + p);
   long long ca, cb;
   const int nctas = pair_ctas(p, prefix, sp, ca, cb);
   const bool single = (nctas == 1);
@@ -223,8 +237,10 @@ __device__ void fused_merge(const FusedArgs& f, float* out, const float* part, i
   }
   if (tid == 0) {
     // commit the pair's new length, used slots and minimum -- once no CTA can still be
-    // reading lengths for its schedule (every CTA counts itself in after building it)
-    bool ready = ld_acquire_gpu(f.ctr) >= (int)gridDim.x;
+    // reading lengths for its schedule (every CTA counts itself in after building it);
+    // the first merge of this CTA to see that tells the later ones through shared memory
+    bool ready = ld_acquire_cta(sched_seen) != 0;
+    if (!ready) ready = ld_acquire_gpu(f.ctr) >= (int)gridDim.x;
     if (!ready) {
       const unsigned long long t0 = globaltimer();
       while (!(ready = ld_acquire_gpu(f.ctr) >= (int)gridDim.x))
@@ -234,7 +250,7 @@ __device__ void fused_merge(const FusedArgs& f, float* out, const float* part, i
         }
     }
     if (ready) {
-      const int4 mt = __ldcg(reinterpret_cast<const int4*>(f.meta_next) + p);
+      st_release_cta(sched_seen, 1);
       st.len[p] = mt.x;
       st.nvalid[p] = mt.y;
       st.min_score[p] = __int_as_float(mt.z);
@@ -648,7 +664,8 @@ __device__ void fused_scorer(const FusedArgs& f, const bf16* q, float* out, cons
       if (!((lm >> r) & 1u)) continue;
       const int pair = (b0 + w + kFusedSW * r) * H + h;
       fused_merge<HD, G, 32>(f, out, part, part_count, pair, prefix, sp, -1, nullptr, nullptr,
-                             nullptr, lane, [] { __syncwarp(); });
+                             nullptr, lane, reinterpret_cast<int*>(fsm + FusedSmem::FLAG),
+                             [] { __syncwarp(); });
     }
     ssync();   // X and the per-sequence state are reused by the next unit
   }
