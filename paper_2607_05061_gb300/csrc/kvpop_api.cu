@@ -348,7 +348,7 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     c->fb.part_c = static_cast<float*>(p);
     if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * 4 * 4); c->fb.meta_next = (int32_t*)p; }
     if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * (2 * dm.G + 2 * d) * 4); c->fb.xtra = (float*)p; }
-    if (s == KVPOP_OK) { s = dev_alloc(c, &p, 16); c->fb.ctr = (int32_t*)p; }
+    if (s == KVPOP_OK) { s = dev_alloc(c, &p, 16); c->fb.ctr = static_cast<unsigned long long*>(p); }
   }
 #undef ALLOC
   // q | k | v staging in one block, so that adjacent host buffers take a single copy

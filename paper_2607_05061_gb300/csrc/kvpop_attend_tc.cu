@@ -177,10 +177,16 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
   build_schedule<NT>(a.nvalid, a.len, npairs, a.B, a.D, TILE, prefix, scan, a.err);
   const long long Ttot = prefix[npairs];
   if constexpr (FUSED) {
-    // lengths and used-slot counts read: their commits may start once every CTA is here
+    // lengths and used-slot counts read: their commits may start once every CTA of this
+    // launch is here.  The count runs on over launches, and a launch's CTAs all start after
+    // the previous launch has ended, so old / grid numbers this launch for each of its CTAs
+    // and the count it must reach is the end of that epoch (kept in shared memory).
     if (tid == 0) {
       __threadfence();
-      atomicAdd(f.ctr, 1);
+      const unsigned long long old = atomicAdd(f.ctr, 1ull);
+      unsigned long long* target = reinterpret_cast<unsigned long long*>(
+          smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::FLAG + 8);
+      *target = (old / gridDim.x + 1) * gridDim.x;
     }
   } else {
     if (Ttot <= 0) return;
@@ -499,17 +505,6 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
   }
   if (cur >= 0) finalize(cur);
   }   // consumers
-  if constexpr (FUSED) {
-    // the last CTA out re-arms the grid counters for the next step
-    __syncthreads();
-    if (tid == 0) {
-      __threadfence();
-      if (atomicAdd(f.ctr + 1, 1) == (int)gridDim.x - 1) {
-        f.ctr[0] = 0;
-        f.ctr[1] = 0;
-      }
-    }
-  }
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

@@ -172,7 +172,7 @@ struct FusedBufs {
   float* part_c;               // [pairs][G d + 2 G]
   int32_t* meta_next;          // [pairs][4]
   float* xtra;                 // [pairs][2 G + 2 d]
-  int32_t* ctr;                // [2], zero between launches
+  unsigned long long* ctr;     // CTAs past their schedule over all launches (zero at init)
 };
 bool tc_fused_ok(const Dims& dm);
 int tc_fused_max_grid();         // largest grid the fused kernel's split table holds

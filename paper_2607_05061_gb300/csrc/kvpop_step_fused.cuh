@@ -39,7 +39,7 @@ struct FusedArgs {
   int32_t* meta_next;              // [pairs][4]: length, used slots, min priority (bits), min slot
   float* xtra;                     // [pairs][2 G + 2 d]: logits of the two changed keys per head
                                    // (log2 domain, -inf when absent), then their V rows
-  int32_t* ctr;                    // [2]: CTAs past their schedule, CTAs finished
+  unsigned long long* ctr;         // CTAs past their schedule, counted over all launches
   int batch, H, F, Fp, s, act;   // Fp: W1 / b1 / w2 row length (F rounded up to 4)
 };
 
@@ -53,7 +53,8 @@ struct FusedSmem {
   static constexpr int SEQ = RP + kFusedSW * kFusedSeqs * 4;   // [4][16] len, nvalid, min, min slot
   static constexpr int SXC = SEQ + 4 * kFusedSeqs * 4;   // [4][2] extra-key logits (consumers)
   static constexpr int SXS = SXC + 32;                   // (spare)
-  static constexpr int FLAG = SXS + kFusedSW * 32;       // int flags: [0] every CTA's schedule built
+  static constexpr int FLAG = SXS + kFusedSW * 32;       // [0] int: every CTA's schedule built;
+                                                         // [8] u64: the count that means it
   static constexpr int BND = FLAG + 16;                  // [kMaxSplit + 1] ints: CTA ranges
   static constexpr int WBAR = BND + (kMaxSplit + 1) * 4 + 4;   // [3] mbarriers of the weight ring
   static constexpr int W1R = (WBAR + 24 + 127) & ~127;   // [3][kW1Rows][Fp] weight ring
@@ -68,6 +69,11 @@ __host__ __device__ inline size_t fused_smem_bytes(int Fp) {
 __device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ unsigned long long ld_acquire_gpu(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 // CTA-scope release / acquire on a shared-memory flag (a fact one warp established
@@ -239,11 +245,12 @@ __device__ void fused_merge(const FusedArgs& f, float* out, const float* part, i
     // commit the pair's new length, used slots and minimum -- once no CTA can still be
     // reading lengths for its schedule (every CTA counts itself in after building it);
     // the first merge of this CTA to see that tells the later ones through shared memory
+    const unsigned long long target = *reinterpret_cast<const unsigned long long*>(sched_seen + 2);
     bool ready = ld_acquire_cta(sched_seen) != 0;
-    if (!ready) ready = ld_acquire_gpu(f.ctr) >= (int)gridDim.x;
+    if (!ready) ready = ld_acquire_gpu(f.ctr) >= target;
     if (!ready) {
       const unsigned long long t0 = globaltimer();
-      while (!(ready = ld_acquire_gpu(f.ctr) >= (int)gridDim.x))
+      while (!(ready = ld_acquire_gpu(f.ctr) >= target))
         if (globaltimer() - t0 > kWaitLimitNs) {
           atomicCAS(st.err, 0, DEVERR_TIMEOUT_SCHED);
           break;
