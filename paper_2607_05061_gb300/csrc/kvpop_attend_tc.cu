@@ -375,6 +375,9 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
       if (tid == 0) *flag = (ld_acquire_gpu(a.part_count + p) == nctas);
       consumer_sync();
       bool last = *flag != 0;
+      // seen as last by the acquire above (ordered for every consumer by the barrier), or
+      // by the relaxed count below, which needs a fence before the others' data is read
+      const bool acquired = last;
       if (!last) {
         float* dst = (nctas == 1) ? f.part_c + (size_t)p * PSTRIDE
                                   : a.part + ((size_t)blockIdx.x * 2 + ((prefix[p] < t0) ? 0 : 1)) * PSTRIDE;
@@ -393,7 +396,7 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
         last = *flag != 0;
       }
       if (last) {
-        __threadfence();
+        if (!acquired) __threadfence();
         fused_merge<HD, G, NCT>(f, a.out, a.part, a.part_count, p, prefix, sp, (long long)blockIdx.x,
                                 om, ol, oo, tid, sched_seen, [] { consumer_sync(); });
       }
