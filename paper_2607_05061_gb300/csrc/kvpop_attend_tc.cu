@@ -199,8 +199,8 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
     if (blockIdx.x >= NC) return;
   }
   // FUSED: a CTA without tiles (or a step without any) still runs its scorer units, and
-  // the CTAs with one scorer unit more than the rest stream 3/64 fewer tiles (when every
-  // CTA has at least 4)
+  // the CTAs with one scorer unit more than the rest stream KVPOP_FUSED_SPLIT_K / 64 fewer
+  // tiles (when every CTA has at least 4)
   int* bnd = reinterpret_cast<int*>(smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::BND);
   int* sched_seen = reinterpret_cast<int*>(smem + Tr::al16(Tr::OFF_PREFIX + (npairs + 1) * 4) + FusedSmem::FLAG);
   Split sp{Ttot, NC, bnd};
