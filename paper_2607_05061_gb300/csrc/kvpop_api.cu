@@ -349,6 +349,10 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * 4 * 4); c->fb.meta_next = (int32_t*)p; }
     if (s == KVPOP_OK) { s = dev_alloc(c, &p, pairs * (2 * dm.G + 2 * d) * 4); c->fb.xtra = (float*)p; }
     if (s == KVPOP_OK) { s = dev_alloc(c, &p, 16); c->fb.ctr = static_cast<unsigned long long*>(p); }
+    if (s == KVPOP_OK) {
+      s = dev_alloc(c, &p, (size_t)c->fused_grid * sizeof(int2));
+      c->fb.start_prev = static_cast<int2*>(p);
+    }
   }
 #undef ALLOC
   // q | k | v staging in one block, so that adjacent host buffers take a single copy
@@ -414,6 +418,8 @@ static kvpop_status init_cache(const kvpop_config* cfg_in, const kvpop_scorer* s
     if (e == cudaSuccess && sc) e = NOTE(cudaMemcpyAsync(b2, sc->b2, H * 4, cudaMemcpyDefault, stream));
     if (e == cudaSuccess && c->use_tf32) e = NOTE(prepare_score_tf32(dm, W1, c->w1t, sc_map_ptr(c), stream));
     if (e == cudaSuccess && c->use_fused) e = NOTE(cudaMemsetAsync(c->fb.ctr, 0, 16, stream));
+    if (e == cudaSuccess && c->use_fused)
+      e = NOTE(cudaMemsetAsync(c->fb.start_prev, 0, (size_t)c->fused_grid * sizeof(int2), stream));
     std::vector<float> minus_inf;
     if (c->mlstm) {
       // mLSTM weights: column blocks of Wcat [2d][NC] = [W_k | W_v | W_q | w_i | w_f | 0]

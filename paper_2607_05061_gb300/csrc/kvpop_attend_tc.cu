@@ -45,6 +45,9 @@ constexpr float kThr = 8.0f;
 #define KVPOP_TC_MINBLOCKS 1
 #endif
 // Fused step: tiles (in 64ths) that a CTA with one scorer unit more than the rest gives up.
+#ifndef KVPOP_FUSED_PREFETCH_TILES
+#define KVPOP_FUSED_PREFETCH_TILES 4
+#endif
 #ifndef KVPOP_FUSED_SPLIT_K
 #define KVPOP_FUSED_SPLIT_K 5
 #endif
@@ -167,6 +170,22 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
     mbar_fence_init();
   }
   if constexpr (FUSED) {
+    // Where this CTA's range began last launch (the split stays the same from step to step
+    // once the cache is full): its first tiles go to L2 now, while the previous step's
+    // slowest CTAs still stream, so that this step starts on L2 hits.  A hint only: L2 is
+    // coherent, and a stale record just prefetches something else within the slots.
+    if (tid == 0 && f.start_prev != nullptr) {
+      const int2 sp = __ldcg(f.start_prev + blockIdx.x);
+      const bf16* sk = static_cast<const bf16*>(f.st.slotK);
+      const bf16* sv = static_cast<const bf16*>(f.st.slotV);
+      for (int k = 0; k < KVPOP_FUSED_PREFETCH_TILES; ++k) {
+        const long long slot = (long long)(sp.y + k) * TILE;
+        if (sp.x < 0 || sp.x >= npairs || sp.y < 0 || slot + TILE > a.B) break;
+        const size_t row = (size_t)sp.x * a.B + (size_t)slot;
+        prefetch_l2(sk + row * HD, (uint32_t)(TILE * HD * 2));
+        prefetch_l2(sv + row * HD, (uint32_t)(TILE * HD * 2));
+      }
+    }
     // the next step's kernel may be scheduled now: it waits for this grid before reading
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   }
@@ -224,6 +243,7 @@ __global__ void __launch_bounds__(FUSED ? TcTraits<HD, G>::THREADS_F : TcTraits<
       if (prefix[mid] <= t0) lo = mid; else hi = mid - 1;
     }
     p0 = lo;
+    if (FUSED && tid == 0 && f.start_prev != nullptr) f.start_prev[blockIdx.x] = make_int2(p0, (int)(t0 - prefix[p0]));
   }
   if constexpr (FUSED) {
     if (warp > NWC) {
@@ -676,6 +696,7 @@ cudaError_t tc_launch_fused(const State& st, const Dims& dm, const void* maps, c
   f.meta_next = fb.meta_next;
   f.xtra = fb.xtra;
   f.ctr = fb.ctr;
+  f.start_prev = fb.start_prev;
   f.batch = dm.batch;
   f.H = dm.H;
   f.F = dm.F;

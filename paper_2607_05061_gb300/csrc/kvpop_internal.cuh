@@ -173,6 +173,7 @@ struct FusedBufs {
   int32_t* meta_next;          // [pairs][4]
   float* xtra;                 // [pairs][2 G + 2 d]
   unsigned long long* ctr;     // CTAs past their schedule over all launches (zero at init)
+  int2* start_prev;            // [grid] where each CTA's range began last launch (zero at init)
 };
 bool tc_fused_ok(const Dims& dm);
 int tc_fused_max_grid();         // largest grid the fused kernel's split table holds

@@ -40,6 +40,8 @@ struct FusedArgs {
   float* xtra;                     // [pairs][2 G + 2 d]: logits of the two changed keys per head
                                    // (log2 domain, -inf when absent), then their V rows
   unsigned long long* ctr;         // CTAs past their schedule, counted over all launches
+  int2* start_prev;                // [grid] (pair, tile of the pair) each CTA's range began
+                                   // with in the last launch
   int batch, H, F, Fp, s, act;   // Fp: W1 / b1 / w2 row length (F rounded up to 4)
 };
 
